@@ -1,0 +1,716 @@
+// engine.cu - the C ABI of libssd (include/ssd.h): handle, buffers, the
+// forward sequence of one decoder step, CUDA-graph capture of the draft step
+// and of the verification step, and the decoding loop of self-speculative
+// decoding (arxiv 2309.08168, Algorithms 1, 2 and 4).
+//
+// Decoding loop, one round (Sec. 3.2):
+//   draft  : K_eff replays of the draft-step graph; each runs the forward of
+//            one token through the sublayers outside the skip set z, writes KV
+//            only in the attention sublayers it runs, and appends d_j;
+//   verify : one replay of the verification graph for M = K_eff + 1 rows
+//            [x_last, d_1 .. d_K_eff] at positions len .. len + K_eff, which
+//            rewrites KV for every layer and ends in the acceptance kernel;
+//   accept : n accepted drafts plus a correction / bonus token are emitted,
+//            len <- len + 1 + n (the KV rollback is this length pointer).
+// Everything between two rounds stays on the device; the host reads one int
+// (tokens emitted so far) per round to size the next round.
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <map>
+#include <string>
+#include <vector>
+
+#include "ssd.h"
+#include "ssd_internal.cuh"
+
+using namespace ssd;
+
+namespace ssd {
+int sampling_configure();
+}
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const std::string& msg) {
+    g_err = msg;
+    return code;
+}
+
+#define CUDA_TRY(expr, what)                                                                    \
+    do {                                                                                        \
+        cudaError_t _e = (cudaError_t)(expr);                                                   \
+        if (_e != cudaSuccess)                                                                  \
+            return fail(SSD_ERR_CUDA, std::string(what) + ": " + cudaGetErrorString(_e));     \
+    } while (0)
+
+// Debug mode (SSD_SYNC_CHECK=1 in the environment at ssd_create): every
+// launch outside graph capture is followed by a stream synchronisation, so a
+// failing kernel is reported by name and layer.
+#define LAUNCH(h, expr, what, layer)                                                            \
+    do {                                                                                        \
+        CUDA_TRY(expr, what);                                                                   \
+        if ((h)->sync_check) {                                                                  \
+            cudaStreamCaptureStatus _cs = cudaStreamCaptureStatusNone;                           \
+            cudaStreamIsCapturing((h)->stream, &_cs);                                           \
+            if (_cs == cudaStreamCaptureStatusNone) {                                           \
+                cudaError_t _s = cudaStreamSynchronize((h)->stream);                            \
+                if (_s != cudaSuccess)                                                          \
+                    return fail(SSD_ERR_CUDA, std::string(what) + " (layer " +                 \
+                                                  std::to_string(layer) + "): " + cudaGetErrorString(_s)); \
+            }                                                                                   \
+        }                                                                                       \
+    } while (0)
+
+struct GemmPlan {
+    int kc = 0, ksplit = 0, n_tiles = 0;
+};
+
+GemmPlan make_plan(int K, int n_tiles) {
+    GemmPlan p;
+    p.kc = K >= 512 ? 512 : ((K + 63) / 64) * 64;
+    p.ksplit = (K + p.kc - 1) / p.kc;
+    p.n_tiles = n_tiles;
+    return p;
+}
+
+enum GraphKind { G_DRAFT = 0, G_VERIFY = 1 };
+
+}  // namespace
+
+struct ssd_handle {
+    ssd_config cfg{};
+    int device = 0;
+    cudaStream_t stream = nullptr;
+    bool own_stream = false;
+
+    const bf16* embed = nullptr;
+    const bf16* final_norm = nullptr;
+    const bf16* lm_head = nullptr;
+    std::vector<const bf16*> wq, wk, wv, wo, attn_norm, w_gate, w_up, w_down, mlp_norm;
+    std::vector<void*> owned;  // weight copies (on_device = 0)
+    std::vector<void*> bufs;   // work buffers
+    std::vector<uint8_t> mask;
+    float temperature = 1.f, top_p = 1.f;
+
+    // device buffers
+    f16* kc = nullptr;   // [L][Hkv][max_seq][hd] fp16
+    f16* vc = nullptr;
+    size_t kv_layer = 0;  // elements per layer of one of K / V
+    float* h = nullptr;
+    float* xb = nullptr;  // normalised rows entering a projection [16][d]
+    float* q = nullptr;
+    float* attn = nullptr;  // attention output [16][H*hd]
+    float* act = nullptr;   // SwiGLU output [16][ffn]
+    float* logits = nullptr;
+    float* p_rows = nullptr;
+    float* q_rows = nullptr;
+    float* partial = nullptr;
+    unsigned* counters = nullptr;  // [gemm tiles | attention kv heads | accept]
+    int gemm_counters = 0;
+    float* attn_part = nullptr;
+    int n_chunks = 0;
+    float2* rope = nullptr;
+    int* tok = nullptr;  // [max_seq] prompt | [16] debug rows
+    int* out = nullptr;  // [max_seq]
+    int* argbuf = nullptr;
+    DecodeState* st = nullptr;
+    DecodeState* st_host = nullptr;  // pinned staging
+    int* emitted_host = nullptr;     // pinned
+
+    GemmPlan p_qkv, p_o, p_gu, p_down, p_head;
+    std::map<int, cudaGraphExec_t> graphs;
+    std::map<int, int> graph_launches;  // kernels per replay
+    std::vector<cudaEvent_t> events;
+
+    bool prefilled = false;
+    int n_prompt = 0;
+    int last_prompt_token = 0;
+    bool sync_check = false;
+};
+
+namespace {
+
+int graph_key(int kind, int M, int mode) { return (mode * 2 + kind) * 64 + M; }
+
+void drop_graphs(ssd_handle* h, int kind) {
+    for (auto it = h->graphs.begin(); it != h->graphs.end();) {
+        if (kind < 0 || ((it->first / 64) % 2) == kind) {
+            cudaGraphExecDestroy(it->second);
+            h->graph_launches.erase(it->first);
+            it = h->graphs.erase(it);
+        } else {
+            ++it;
+        }
+    }
+}
+
+// The forward of one decoder step over M rows: embedding, the sublayers that
+// run (all of them, or those outside the skip set when draft), final norm and
+// lm_head.  Launches only; no host synchronisation (graph-capturable).
+int forward(ssd_handle* h, int M, int src, const int* toks, int pos0, bool draft, bool logits,
+            int* n_launch = nullptr, bool gemm_only = false) {
+    const ssd_config& c = h->cfg;
+    const int d = c.d_model, qd = c.n_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
+    cudaStream_t s = h->stream;
+    int launched = 0;
+    const bool aux = !gemm_only;  // norms, embedding, attention
+    if (aux) { LAUNCH(h, launch_embed(h->embed, d, M, src, toks, pos0, h->st, h->h, s), "embed", -1); ++launched; }
+    for (int l = 0; l < c.n_layers; ++l) {
+        const bool run_a = !(draft && h->mask[2 * l]);
+        const bool run_m = !(draft && h->mask[2 * l + 1]);
+        if (run_a) {
+            if (aux) { LAUNCH(h, launch_rmsnorm(h->h, h->attn_norm[l], d, M, c.rms_eps, h->xb, s), "rmsnorm", l); ++launched; }
+            GemmArgs a{};
+            a.w0 = h->wq[l]; a.w1 = h->wk[l]; a.w2 = h->wv[l];
+            a.N = qd + 2 * kvd; a.K = d;
+            a.kc = h->p_qkv.kc; a.ksplit = h->p_qkv.ksplit; a.n_tiles = h->p_qkv.n_tiles;
+            a.x = h->xb; a.M = M; a.partial = h->partial; a.counters = h->counters;
+            a.n_heads = c.n_heads; a.n_kv_heads = c.n_kv_heads; a.head_dim = c.head_dim;
+            a.max_seq = c.max_seq; a.q_out = h->q;
+            a.k_cache = h->kc + (size_t)l * h->kv_layer;
+            a.v_cache = h->vc + (size_t)l * h->kv_layer;
+            a.rope = h->rope; a.st = h->st; a.err = &h->st->err;
+            LAUNCH(h, launch_gemm(EPI_QKV, a, s), "qkv projection", l);
+            ++launched;
+            AttnArgs t{};
+            t.q = h->q; t.k_cache = a.k_cache; t.v_cache = a.v_cache; t.out = h->attn;
+            t.part = h->attn_part; t.counters = h->counters + h->gemm_counters;
+            t.M = M; t.n_heads = c.n_heads; t.n_kv_heads = c.n_kv_heads; t.head_dim = c.head_dim;
+            t.max_seq = c.max_seq; t.n_chunks = h->n_chunks;
+            t.scale = 1.0f / std::sqrt((float)c.head_dim); t.st = h->st; t.err = &h->st->err;
+            if (aux) { LAUNCH(h, launch_attention(t, s), "attention", l); ++launched; }
+            GemmArgs o{};
+            o.w0 = h->wo[l]; o.N = d; o.K = qd;
+            o.kc = h->p_o.kc; o.ksplit = h->p_o.ksplit; o.n_tiles = h->p_o.n_tiles;
+            o.x = h->attn; o.M = M; o.partial = h->partial; o.counters = h->counters;
+            o.out_f32 = h->h; o.ldo = d; o.st = h->st; o.err = &h->st->err;
+            LAUNCH(h, launch_gemm(EPI_RESID, o, s), "output projection", l);
+            ++launched;
+        }
+        if (run_m) {
+            if (aux) { LAUNCH(h, launch_rmsnorm(h->h, h->mlp_norm[l], d, M, c.rms_eps, h->xb, s), "rmsnorm", l); ++launched; }
+            GemmArgs g{};
+            g.w0 = h->w_gate[l]; g.w1 = h->w_up[l]; g.N = 2 * c.ffn; g.K = d;
+            g.kc = h->p_gu.kc; g.ksplit = h->p_gu.ksplit; g.n_tiles = h->p_gu.n_tiles;
+            g.x = h->xb; g.M = M; g.partial = h->partial; g.counters = h->counters;
+            g.out_act = h->act; g.ffn = c.ffn; g.st = h->st; g.err = &h->st->err;
+            LAUNCH(h, launch_gemm(EPI_SWIGLU, g, s), "gate/up projection", l);
+            ++launched;
+            GemmArgs w{};
+            w.w0 = h->w_down[l]; w.N = d; w.K = c.ffn;
+            w.kc = h->p_down.kc; w.ksplit = h->p_down.ksplit; w.n_tiles = h->p_down.n_tiles;
+            w.x = h->act; w.M = M; w.partial = h->partial; w.counters = h->counters;
+            w.out_f32 = h->h; w.ldo = d; w.st = h->st; w.err = &h->st->err;
+            LAUNCH(h, launch_gemm(EPI_RESID, w, s), "down projection", l);
+            ++launched;
+        }
+    }
+    if (logits) {
+        if (aux) { LAUNCH(h, launch_rmsnorm(h->h, h->final_norm, d, M, c.rms_eps, h->xb, s), "final norm", -1); ++launched; }
+        GemmArgs o{};
+        o.w0 = h->lm_head; o.N = c.vocab; o.K = d;
+        o.kc = h->p_head.kc; o.ksplit = h->p_head.ksplit; o.n_tiles = h->p_head.n_tiles;
+        o.x = h->xb; o.M = M; o.partial = h->partial; o.counters = h->counters;
+        o.out_f32 = h->logits; o.ldo = c.vocab; o.st = h->st; o.err = &h->st->err;
+        LAUNCH(h, launch_gemm(EPI_LOGITS, o, s), "lm_head", -1);
+        ++launched;
+    }
+    if (n_launch) *n_launch = launched;
+    return SSD_OK;
+}
+
+// Weight bytes one forward streams (bf16): the matrices and norm gains of
+// every sublayer that runs, one embedding row, the final norm and lm_head.
+double forward_weight_bytes(const ssd_handle* h, bool draft, bool gemm_only) {
+    const ssd_config& c = h->cfg;
+    const double d = c.d_model, qd = (double)c.n_heads * c.head_dim, kvd = (double)c.n_kv_heads * c.head_dim;
+    const double attn = (qd * d + 2 * kvd * d + d * qd) * 2 + (gemm_only ? 0 : d * 2);
+    const double mlp = 3.0 * c.ffn * d * 2 + (gemm_only ? 0 : d * 2);
+    double b = (double)c.vocab * d * 2 + (gemm_only ? 0 : 2 * d * 2);
+    for (int l = 0; l < c.n_layers; ++l) {
+        if (!(draft && h->mask[2 * l])) b += attn;
+        if (!(draft && h->mask[2 * l + 1])) b += mlp;
+    }
+    return b;
+}
+
+unsigned* accept_counter(ssd_handle* h) { return h->counters + h->gemm_counters + h->cfg.n_kv_heads; }
+
+int step_launches(ssd_handle* h, int kind, int M, int mode, int* n_launch) {
+    const int V = h->cfg.vocab;
+    int n = 0;
+    if (kind == G_DRAFT) {
+        int rc = forward(h, 1, SRC_DRAFT, nullptr, 0, true, true, &n);
+        if (rc) return rc;
+        *n_launch = n + 1;
+        if (mode == SSD_GREEDY) CUDA_TRY(launch_greedy_draft(h->logits, V, h->st, h->stream), "draft argmax");
+        else CUDA_TRY(launch_sample_draft(h->logits, V, h->st, h->q_rows, h->stream), "draft sample");
+        return SSD_OK;
+    }
+    int rc = forward(h, M, SRC_VERIFY, nullptr, 0, false, true, &n);
+    if (rc) return rc;
+    *n_launch = n + 1;
+    if (mode == SSD_GREEDY)
+        CUDA_TRY(launch_greedy_accept(h->logits, V, M, h->st, h->out, accept_counter(h), h->argbuf,
+                                      h->stream), "greedy accept");
+    else
+        CUDA_TRY(launch_sample_accept(h->logits, V, M, h->st, h->p_rows, h->q_rows, h->out,
+                                      accept_counter(h), h->stream), "sample accept");
+    return SSD_OK;
+}
+
+int get_graph(ssd_handle* h, int kind, int M, int mode, cudaGraphExec_t* out, int* n_launch) {
+    const int key = graph_key(kind, M, mode);
+    auto it = h->graphs.find(key);
+    if (it != h->graphs.end()) {
+        *out = it->second;
+        *n_launch = h->graph_launches[key];
+        return SSD_OK;
+    }
+    cudaGraph_t g = nullptr;
+    CUDA_TRY(cudaStreamBeginCapture(h->stream, cudaStreamCaptureModeThreadLocal), "begin capture");
+    int rc = step_launches(h, kind, M, mode, n_launch);
+    cudaError_t e = cudaStreamEndCapture(h->stream, &g);
+    if (rc) { if (g) cudaGraphDestroy(g); return rc; }
+    CUDA_TRY(e, "end capture");
+    cudaGraphExec_t exec = nullptr;
+    e = cudaGraphInstantiate(&exec, g, 0);
+    cudaGraphDestroy(g);
+    CUDA_TRY(e, "graph instantiate");
+    h->graphs[key] = exec;
+    h->graph_launches[key] = *n_launch;
+    *out = exec;
+    return SSD_OK;
+}
+
+template <typename T>
+int dalloc(ssd_handle* h, T** p, size_t n, std::vector<void*>* track) {
+    (void)h;
+    void* v = nullptr;
+    cudaError_t e = cudaMalloc(&v, n * sizeof(T) + 16);
+    if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(SSD_ERR_OOM, std::string("cudaMalloc failed: ") + cudaGetErrorString(e));
+    }
+    track->push_back(v);
+    *p = (T*)v;
+    return SSD_OK;
+}
+
+void free_all(ssd_handle* h, std::vector<void*>& v) {
+    for (void* p : v) cudaFree(p);
+    v.clear();
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+int check_config(const ssd_config* c) {
+    if (!c) return fail(SSD_ERR_INVALID_ARG, "config is NULL");
+    if (c->n_layers < 1 || c->d_model < 64 || c->d_model % 64)
+        return fail(SSD_ERR_INVALID_ARG, "n_layers >= 1 and d_model a positive multiple of 64 required");
+    if (c->head_dim != 64 && c->head_dim != 128)
+        return fail(SSD_ERR_INVALID_ARG, "head_dim must be 64 or 128");
+    if (c->n_heads < 1 || c->n_kv_heads < 1 || c->n_heads % c->n_kv_heads)
+        return fail(SSD_ERR_INVALID_ARG, "n_heads must be a positive multiple of n_kv_heads");
+    if (c->ffn < 16 || c->ffn % 16) return fail(SSD_ERR_INVALID_ARG, "ffn must be a positive multiple of 16");
+    if (c->vocab < 2 || c->vocab > 32768) return fail(SSD_ERR_INVALID_ARG, "vocab must be in [2, 32768]");
+    if (c->max_seq < 2 || c->max_seq > (1 << 24)) return fail(SSD_ERR_INVALID_ARG, "max_seq out of range");
+    if (!(c->rms_eps > 0.f) || !(c->rope_theta > 0.f))
+        return fail(SSD_ERR_INVALID_ARG, "rms_eps and rope_theta must be positive");
+    const int G = c->n_heads / c->n_kv_heads;
+    size_t attn_smem = 2 * kAttnChunk * (c->head_dim * 2 + 16) + (size_t)G * kMaxRows * c->head_dim * 4 +
+                       8 * kAttnChunk * 4;
+    if (attn_smem > 200 * 1024) return fail(SSD_ERR_INVALID_ARG, "n_heads / n_kv_heads too large");
+    return SSD_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* ssd_last_error(void) { return g_err.c_str(); }
+
+void ssd_destroy(ssd_handle* h) {
+    if (!h) return;
+    cudaSetDevice(h->device);
+    if (h->stream) cudaStreamSynchronize(h->stream);
+    drop_graphs(h, -1);
+    for (cudaEvent_t e : h->events) cudaEventDestroy(e);
+    free_all(h, h->bufs);
+    free_all(h, h->owned);
+    if (h->st_host) cudaFreeHost(h->st_host);
+    if (h->emitted_host) cudaFreeHost(h->emitted_host);
+    if (h->own_stream && h->stream) cudaStreamDestroy(h->stream);
+    delete h;
+}
+
+int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, ssd_handle** out) {
+    if (!out) return fail(SSD_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    int rc = check_config(cfg);
+    if (rc) return rc;
+    if (!w || !w->embed || !w->final_norm || !w->lm_head || !w->wq || !w->wk || !w->wv || !w->wo ||
+        !w->attn_norm || !w->w_gate || !w->w_up || !w->w_down || !w->mlp_norm)
+        return fail(SSD_ERR_INVALID_ARG, "weights: NULL member");
+    if (w->on_device != 0 && w->on_device != 1) return fail(SSD_ERR_INVALID_ARG, "weights.on_device must be 0 or 1");
+    const ssd_config c = *cfg;
+    const int L = c.n_layers, d = c.d_model, qd = c.n_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
+    for (int l = 0; l < L; ++l)
+        if (!w->wq[l] || !w->wk[l] || !w->wv[l] || !w->wo[l] || !w->attn_norm[l] || !w->w_gate[l] ||
+            !w->w_up[l] || !w->w_down[l] || !w->mlp_norm[l])
+            return fail(SSD_ERR_INVALID_ARG, "weights: NULL layer tensor");
+
+    ssd_handle* h = new ssd_handle();
+    h->cfg = c;
+    {
+        const char* sc = std::getenv("SSD_SYNC_CHECK");
+        h->sync_check = sc && sc[0] == '1';
+    }
+    cudaGetDevice(&h->device);
+    auto bail = [&](int code) { ssd_destroy(h); return code; };
+    if (cuda_stream) {
+        h->stream = (cudaStream_t)cuda_stream;
+    } else {
+        cudaError_t e = cudaStreamCreateWithFlags(&h->stream, cudaStreamNonBlocking);
+        if (e != cudaSuccess) return bail(fail(SSD_ERR_CUDA, std::string("stream: ") + cudaGetErrorString(e)));
+        h->own_stream = true;
+    }
+    {
+        int e1 = gemm_configure(), e2 = attention_configure(), e3 = sampling_configure();
+        int e = e1 ? e1 : (e2 ? e2 : e3);
+        if (e) return bail(fail(SSD_ERR_CUDA, std::string("kernel setup: ") + cudaGetErrorString((cudaError_t)e)));
+    }
+
+    // weights: borrow device pointers or copy host tensors
+    auto take = [&](const void* src, size_t elems, const bf16** dst) -> int {
+        if (w->on_device) {
+            if (!aligned16(src)) return fail(SSD_ERR_INVALID_ARG, "device weight pointer not 16-byte aligned");
+            *dst = (const bf16*)src;
+            return SSD_OK;
+        }
+        bf16* p = nullptr;
+        int r = dalloc(h, &p, elems, &h->owned);
+        if (r) return r;
+        cudaError_t e = cudaMemcpy(p, src, elems * 2, cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) return fail(SSD_ERR_CUDA, std::string("weight copy: ") + cudaGetErrorString(e));
+        *dst = p;
+        return SSD_OK;
+    };
+    const size_t V = c.vocab, F = c.ffn;
+    if ((rc = take(w->embed, V * d, &h->embed)) || (rc = take(w->final_norm, d, &h->final_norm)) ||
+        (rc = take(w->lm_head, V * d, &h->lm_head)))
+        return bail(rc);
+    h->wq.resize(L); h->wk.resize(L); h->wv.resize(L); h->wo.resize(L); h->attn_norm.resize(L);
+    h->w_gate.resize(L); h->w_up.resize(L); h->w_down.resize(L); h->mlp_norm.resize(L);
+    for (int l = 0; l < L; ++l) {
+        if ((rc = take(w->wq[l], (size_t)qd * d, &h->wq[l])) || (rc = take(w->wk[l], (size_t)kvd * d, &h->wk[l])) ||
+            (rc = take(w->wv[l], (size_t)kvd * d, &h->wv[l])) || (rc = take(w->wo[l], (size_t)d * qd, &h->wo[l])) ||
+            (rc = take(w->attn_norm[l], d, &h->attn_norm[l])) ||
+            (rc = take(w->w_gate[l], F * d, &h->w_gate[l])) || (rc = take(w->w_up[l], F * d, &h->w_up[l])) ||
+            (rc = take(w->w_down[l], (size_t)d * F, &h->w_down[l])) ||
+            (rc = take(w->mlp_norm[l], d, &h->mlp_norm[l])))
+            return bail(rc);
+    }
+    h->mask.assign(2 * L, 0);
+
+    // plans
+    h->p_qkv = make_plan(d, (qd + 2 * kvd) / kTileRows);
+    h->p_o = make_plan(qd, (d + kTileRows - 1) / kTileRows);
+    h->p_gu = make_plan(d, (c.ffn + 31) / 32);
+    h->p_down = make_plan(c.ffn, (d + kTileRows - 1) / kTileRows);
+    h->p_head = make_plan(d, (c.vocab + kTileRows - 1) / kTileRows);
+    size_t part = 0;
+    int tiles = 0;
+    for (const GemmPlan* p : {&h->p_qkv, &h->p_o, &h->p_gu, &h->p_down, &h->p_head}) {
+        part = std::max(part, (size_t)p->ksplit * kMaxRows * p->n_tiles * kTileRows);
+        tiles = std::max(tiles, p->n_tiles);
+    }
+    h->gemm_counters = tiles;
+    h->n_chunks = (c.max_seq + kAttnChunk - 1) / kAttnChunk;
+    const int G = c.n_heads / c.n_kv_heads;
+
+    // buffers
+    std::vector<void*>& B = h->bufs;
+    h->kv_layer = (size_t)c.n_kv_heads * c.max_seq * c.head_dim;
+    const size_t HD = c.head_dim;
+    if ((rc = dalloc(h, &h->kc, h->kv_layer * L, &B)) || (rc = dalloc(h, &h->vc, h->kv_layer * L, &B)) ||
+        (rc = dalloc(h, &h->h, (size_t)kMaxRows * d, &B)) || (rc = dalloc(h, &h->xb, (size_t)kMaxRows * d, &B)) ||
+        (rc = dalloc(h, &h->q, (size_t)kMaxRows * qd, &B)) || (rc = dalloc(h, &h->attn, (size_t)kMaxRows * qd, &B)) ||
+        (rc = dalloc(h, &h->act, (size_t)kMaxRows * F, &B)) ||
+        (rc = dalloc(h, &h->logits, (size_t)kMaxRows * V, &B)) ||
+        (rc = dalloc(h, &h->p_rows, (size_t)kMaxRows * V, &B)) ||
+        (rc = dalloc(h, &h->q_rows, (size_t)kMaxRows * V, &B)) || (rc = dalloc(h, &h->partial, part, &B)) ||
+        (rc = dalloc(h, &h->counters, (size_t)tiles + c.n_kv_heads + 4, &B)) ||
+        (rc = dalloc(h, &h->attn_part, (size_t)c.n_kv_heads * h->n_chunks * G * kMaxRows * (HD + 2), &B)) ||
+        (rc = dalloc(h, &h->rope, (size_t)c.max_seq * (HD / 2), &B)) ||
+        (rc = dalloc(h, &h->tok, (size_t)c.max_seq + kMaxRows, &B)) ||
+        (rc = dalloc(h, &h->out, (size_t)c.max_seq, &B)) || (rc = dalloc(h, &h->argbuf, 32, &B)) ||
+        (rc = dalloc(h, &h->st, 1, &B)))
+        return bail(rc);
+    {
+        cudaError_t e = cudaMallocHost(&h->st_host, sizeof(DecodeState));
+        if (e == cudaSuccess) e = cudaMallocHost(&h->emitted_host, sizeof(int) * 4);
+        if (e != cudaSuccess) return bail(fail(SSD_ERR_OOM, "pinned host allocation failed"));
+    }
+    // RoPE table (cos, sin) of pos * theta^(-2i/hd), computed in double
+    {
+        std::vector<float2> tab((size_t)c.max_seq * (HD / 2));
+        for (int p = 0; p < c.max_seq; ++p)
+            for (size_t i = 0; i < HD / 2; ++i) {
+                double a = p * std::pow((double)c.rope_theta, -(2.0 * (double)i) / (double)HD);
+                tab[(size_t)p * (HD / 2) + i] = make_float2((float)std::cos(a), (float)std::sin(a));
+            }
+        cudaError_t e = cudaMemcpy(h->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) return bail(fail(SSD_ERR_CUDA, std::string("rope table: ") + cudaGetErrorString(e)));
+    }
+    cudaError_t e = cudaMemsetAsync(h->counters, 0, ((size_t)tiles + c.n_kv_heads + 4) * sizeof(unsigned), h->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(h->st, 0, sizeof(DecodeState), h->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(h->kc, 0, h->kv_layer * L * sizeof(f16), h->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(h->vc, 0, h->kv_layer * L * sizeof(f16), h->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
+    if (e != cudaSuccess) return bail(fail(SSD_ERR_CUDA, std::string("init: ") + cudaGetErrorString(e)));
+    *out = h;
+    return SSD_OK;
+}
+
+int ssd_set_skip(ssd_handle* h, const uint8_t* mask, int n_sublayers) {
+    if (!h || !mask) return fail(SSD_ERR_INVALID_ARG, "NULL handle or mask");
+    if (n_sublayers != 2 * h->cfg.n_layers) return fail(SSD_ERR_INVALID_ARG, "n_sublayers must be 2 * n_layers");
+    for (int i = 0; i < n_sublayers; ++i)
+        if (mask[i] > 1) return fail(SSD_ERR_INVALID_ARG, "mask values must be 0 or 1");
+    h->mask.assign(mask, mask + n_sublayers);
+    drop_graphs(h, G_DRAFT);
+    return SSD_OK;
+}
+
+int ssd_set_sampling(ssd_handle* h, float temperature, float top_p) {
+    if (!h) return fail(SSD_ERR_INVALID_ARG, "NULL handle");
+    if (!(temperature > 0.f) || !(top_p > 0.f) || top_p > 1.f)
+        return fail(SSD_ERR_INVALID_ARG, "temperature > 0 and 0 < top_p <= 1 required");
+    h->temperature = temperature;
+    h->top_p = top_p;
+    return SSD_OK;
+}
+
+int ssd_prefill(ssd_handle* h, const int32_t* prompt, int n_prompt) {
+    if (!h || !prompt) return fail(SSD_ERR_INVALID_ARG, "NULL handle or prompt");
+    if (n_prompt < 1) return fail(SSD_ERR_INVALID_ARG, "n_prompt must be >= 1");
+    if (n_prompt > h->cfg.max_seq) return fail(SSD_ERR_CAPACITY, "prompt longer than max_seq");
+    for (int i = 0; i < n_prompt; ++i)
+        if (prompt[i] < 0 || prompt[i] >= h->cfg.vocab) return fail(SSD_ERR_INVALID_ARG, "prompt token out of range");
+    CUDA_TRY(cudaSetDevice(h->device), "set device");
+    h->prefilled = false;
+    if (n_prompt > 1)
+        CUDA_TRY(cudaMemcpyAsync(h->tok, prompt, sizeof(int) * (n_prompt - 1), cudaMemcpyHostToDevice, h->stream),
+                 "prompt upload");
+    for (int p0 = 0; p0 < n_prompt - 1; p0 += kMaxRows) {
+        int M = std::min(kMaxRows, n_prompt - 1 - p0);
+        int rc = forward(h, M, SRC_TOKENS, h->tok + p0, p0, false, false);
+        if (rc) return rc;
+    }
+    CUDA_TRY(cudaStreamSynchronize(h->stream), "prefill");
+#ifdef SSD_CHECKED
+    {
+        int derr = 0;
+        CUDA_TRY(cudaMemcpy(&derr, &h->st->err, sizeof(int), cudaMemcpyDeviceToHost), "error flag");
+        if (derr) return fail(SSD_ERR_CUDA, "device check failed with code " + std::to_string(derr));
+    }
+#endif
+    h->prefilled = true;
+    h->n_prompt = n_prompt;
+    h->last_prompt_token = prompt[n_prompt - 1];
+    return SSD_OK;
+}
+
+int ssd_generate(ssd_handle* h, const int32_t* prompt, int n_prompt, int n_new, int K, ssd_mode mode,
+                 uint64_t seed, int32_t* out_tokens, ssd_stats* stats) {
+    if (!h) return fail(SSD_ERR_INVALID_ARG, "NULL handle");
+    if (n_new < 0 || K < 0 || K > kMaxK) return fail(SSD_ERR_INVALID_ARG, "need n_new >= 0 and 0 <= K <= 15");
+    if (mode != SSD_GREEDY && mode != SSD_SAMPLE) return fail(SSD_ERR_INVALID_ARG, "bad mode");
+    if (n_new > 0 && !out_tokens) return fail(SSD_ERR_INVALID_ARG, "out_tokens is NULL");
+    if (prompt) {
+        int rc = ssd_prefill(h, prompt, n_prompt);
+        if (rc) return rc;
+    } else if (!h->prefilled) {
+        return fail(SSD_ERR_STATE, "no prompt given and nothing prefilled");
+    }
+    if (h->n_prompt + n_new > h->cfg.max_seq) return fail(SSD_ERR_CAPACITY, "n_prompt + n_new exceeds max_seq");
+    CUDA_TRY(cudaSetDevice(h->device), "set device");
+    if (stats) std::memset(stats, 0, sizeof(*stats));
+    if (n_new == 0) return SSD_OK;
+
+    DecodeState* init = h->st_host;
+    std::memset(init, 0, sizeof(DecodeState));
+    init->len = h->n_prompt - 1;
+    init->x_last = h->last_prompt_token;
+    init->mode = (int)mode;
+    init->inv_temperature = 1.0f / h->temperature;
+    init->top_p = h->top_p;
+    init->seed = (unsigned long long)seed;
+    CUDA_TRY(cudaMemcpyAsync(h->st, init, sizeof(DecodeState), cudaMemcpyHostToDevice, h->stream), "state upload");
+
+    // graphs needed by this call (captured once, replayed every round)
+    cudaGraphExec_t g_draft = nullptr;
+    int draft_launches = 0;
+    long long launches = 0;
+    if (K > 0) {
+        int rc = get_graph(h, G_DRAFT, 1, mode, &g_draft, &draft_launches);
+        if (rc) return rc;
+    }
+    const size_t need_events = 3 * (size_t)n_new + 2;
+    while (h->events.size() < need_events) {
+        cudaEvent_t ev;
+        CUDA_TRY(cudaEventCreate(&ev), "event create");
+        h->events.push_back(ev);
+    }
+    CUDA_TRY(cudaEventRecord(h->events[0], h->stream), "event");
+    int emitted = 0, round = 0;
+    while (emitted < n_new) {
+        const int Kd = std::min(K, n_new - emitted - 1);
+        cudaGraphExec_t g_verify = nullptr;
+        int verify_launches = 0;
+        int rc = get_graph(h, G_VERIFY, Kd + 1, mode, &g_verify, &verify_launches);
+        if (rc) return rc;
+        launches += (long long)Kd * draft_launches + verify_launches;
+        cudaEvent_t* ev = &h->events[2 + 3 * (size_t)round];
+        CUDA_TRY(cudaEventRecord(ev[0], h->stream), "event");
+        for (int j = 0; j < Kd; ++j) CUDA_TRY(cudaGraphLaunch(g_draft, h->stream), "draft step");
+        CUDA_TRY(cudaEventRecord(ev[1], h->stream), "event");
+        CUDA_TRY(cudaGraphLaunch(g_verify, h->stream), "verification step");
+        CUDA_TRY(cudaEventRecord(ev[2], h->stream), "event");
+        CUDA_TRY(cudaMemcpyAsync(h->emitted_host, &h->st->emitted, sizeof(int), cudaMemcpyDeviceToHost, h->stream),
+                 "state read");
+        CUDA_TRY(cudaStreamSynchronize(h->stream), "round");
+        const int e = *h->emitted_host;
+        if (e <= emitted || e > n_new) return fail(SSD_ERR_CUDA, "decode state corrupted");
+        emitted = e;
+        ++round;
+    }
+    CUDA_TRY(cudaEventRecord(h->events[1], h->stream), "event");
+    CUDA_TRY(cudaMemcpyAsync(out_tokens, h->out, sizeof(int) * n_new, cudaMemcpyDeviceToHost, h->stream), "tokens");
+    CUDA_TRY(cudaMemcpyAsync(h->st_host, h->st, sizeof(DecodeState), cudaMemcpyDeviceToHost, h->stream), "stats");
+    CUDA_TRY(cudaStreamSynchronize(h->stream), "generate");
+    if (stats) {
+        const DecodeState* s = h->st_host;
+        stats->rounds = s->rounds;
+        stats->drafted = s->drafted;
+        stats->accepted = s->accepted;
+        stats->emitted = s->emitted;
+        stats->accept_rate = s->drafted ? (double)s->accepted / s->drafted : 0.0;
+        for (int i = 0; i < 33; ++i) stats->hist[i] = s->hist[i];
+        float dm = 0.f, vm = 0.f, t = 0.f;
+        for (int r = 0; r < round; ++r) {
+            cudaEvent_t* ev = &h->events[2 + 3 * (size_t)r];
+            float a = 0.f, b = 0.f;
+            cudaEventElapsedTime(&a, ev[0], ev[1]);
+            cudaEventElapsedTime(&b, ev[1], ev[2]);
+            dm += a;
+            vm += b;
+        }
+        cudaEventElapsedTime(&t, h->events[0], h->events[1]);
+        stats->draft_ms = dm;
+        stats->verify_ms = vm;
+        stats->total_ms = t;
+        stats->kernel_launches = launches;
+    }
+    return SSD_OK;
+}
+
+int ssd_debug_forward(ssd_handle* h, int draft, const int32_t* tokens, int n_rows, int pos0, float* logits_out) {
+    if (!h || !tokens || !logits_out) return fail(SSD_ERR_INVALID_ARG, "NULL argument");
+    if (n_rows < 1 || n_rows > kMaxRows) return fail(SSD_ERR_INVALID_ARG, "n_rows must be in [1, 16]");
+    if (pos0 < 0 || pos0 + n_rows > h->cfg.max_seq) return fail(SSD_ERR_CAPACITY, "positions beyond max_seq");
+    for (int i = 0; i < n_rows; ++i)
+        if (tokens[i] < 0 || tokens[i] >= h->cfg.vocab) return fail(SSD_ERR_INVALID_ARG, "token out of range");
+    CUDA_TRY(cudaSetDevice(h->device), "set device");
+    int* dt = h->tok + h->cfg.max_seq;
+    CUDA_TRY(cudaMemcpyAsync(dt, tokens, sizeof(int) * n_rows, cudaMemcpyHostToDevice, h->stream), "upload");
+    int rc = forward(h, n_rows, SRC_TOKENS, dt, pos0, draft != 0, true);
+    if (rc) return rc;
+    CUDA_TRY(cudaMemcpyAsync(logits_out, h->logits, sizeof(float) * n_rows * h->cfg.vocab,
+                             cudaMemcpyDeviceToHost, h->stream), "logits");
+    CUDA_TRY(cudaStreamSynchronize(h->stream), "debug forward");
+    return SSD_OK;
+}
+
+int ssd_debug_time_forward(ssd_handle* h, int draft, int rows, int gemm_only, int reps, float* ms_per_forward,
+                           int* launches, double* weight_bytes) {
+    if (!h || !ms_per_forward || !launches || !weight_bytes) return fail(SSD_ERR_INVALID_ARG, "NULL argument");
+    if (rows < 1 || rows > kMaxRows || reps < 1 || rows > h->cfg.max_seq)
+        return fail(SSD_ERR_INVALID_ARG, "rows in [1, 16] and reps >= 1 required");
+    CUDA_TRY(cudaSetDevice(h->device), "set device");
+    const int pos0 = h->cfg.max_seq - rows;
+    int* dt = h->tok + h->cfg.max_seq;
+    CUDA_TRY(cudaMemsetAsync(dt, 0, sizeof(int) * rows, h->stream), "tokens");
+    DecodeState* init = h->st_host;
+    std::memset(init, 0, sizeof(DecodeState));
+    init->pos0 = pos0;
+    CUDA_TRY(cudaMemcpyAsync(h->st, init, sizeof(DecodeState), cudaMemcpyHostToDevice, h->stream), "state");
+    cudaGraph_t g = nullptr;
+    int n = 0;
+    CUDA_TRY(cudaStreamBeginCapture(h->stream, cudaStreamCaptureModeThreadLocal), "begin capture");
+    int rc = forward(h, rows, SRC_TOKENS, dt, pos0, draft != 0, true, &n, gemm_only != 0);
+    cudaError_t e = cudaStreamEndCapture(h->stream, &g);
+    if (rc) { if (g) cudaGraphDestroy(g); return rc; }
+    CUDA_TRY(e, "end capture");
+    cudaGraphExec_t exec = nullptr;
+    e = cudaGraphInstantiate(&exec, g, 0);
+    cudaGraphDestroy(g);
+    CUDA_TRY(e, "graph instantiate");
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    e = cudaEventCreate(&e0);
+    if (e == cudaSuccess) e = cudaEventCreate(&e1);
+    if (e == cudaSuccess) e = cudaGraphLaunch(exec, h->stream);  // warm-up
+    if (e == cudaSuccess) e = cudaEventRecord(e0, h->stream);
+    for (int r = 0; r < reps && e == cudaSuccess; ++r) e = cudaGraphLaunch(exec, h->stream);
+    if (e == cudaSuccess) e = cudaEventRecord(e1, h->stream);
+    if (e == cudaSuccess) e = cudaEventSynchronize(e1);
+    float ms = 0.f;
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, e0, e1);
+    if (e0) cudaEventDestroy(e0);
+    if (e1) cudaEventDestroy(e1);
+    cudaGraphExecDestroy(exec);
+    CUDA_TRY(e, "timing");
+    *ms_per_forward = ms / reps;
+    *launches = n;
+    *weight_bytes = forward_weight_bytes(h, draft != 0, gemm_only != 0);
+    if (pos0 < h->n_prompt) h->prefilled = false;  // the prompt's KV was overwritten
+    return SSD_OK;
+}
+
+int ssd_debug_spec_accept(ssd_handle* h, const float* p, const float* q, int Kd, const int32_t* drafts,
+                          const uint64_t* seeds, int trials, int pos0, int32_t* out) {
+    if (!h || !p || !q || !drafts || !seeds || !out) return fail(SSD_ERR_INVALID_ARG, "NULL argument");
+    if (Kd < 1 || Kd > kMaxK || trials < 1 || pos0 < 0) return fail(SSD_ERR_INVALID_ARG, "bad Kd / trials / pos0");
+    const int V = h->cfg.vocab;
+    for (size_t i = 0; i < (size_t)trials * Kd; ++i)
+        if (drafts[i] < 0 || drafts[i] >= V) return fail(SSD_ERR_INVALID_ARG, "draft token out of range");
+    CUDA_TRY(cudaSetDevice(h->device), "set device");
+    std::vector<void*> tmp;
+    float *dp = nullptr, *dq = nullptr;
+    int *dd = nullptr, *dout = nullptr;
+    unsigned long long* ds = nullptr;
+    int rc = 0;
+    if ((rc = dalloc(h, &dp, (size_t)(Kd + 1) * V, &tmp)) || (rc = dalloc(h, &dq, (size_t)Kd * V, &tmp)) ||
+        (rc = dalloc(h, &dd, (size_t)trials * Kd, &tmp)) || (rc = dalloc(h, &ds, (size_t)trials, &tmp)) ||
+        (rc = dalloc(h, &dout, (size_t)2 * trials, &tmp))) {
+        free_all(h, tmp);
+        return rc;
+    }
+    cudaError_t e = cudaMemcpyAsync(dp, p, sizeof(float) * (Kd + 1) * V, cudaMemcpyHostToDevice, h->stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(dq, q, sizeof(float) * Kd * V, cudaMemcpyHostToDevice, h->stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(dd, drafts, sizeof(int) * trials * Kd, cudaMemcpyHostToDevice, h->stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(ds, seeds, sizeof(uint64_t) * trials, cudaMemcpyHostToDevice, h->stream);
+    if (e == cudaSuccess)
+        e = (cudaError_t)launch_spec_accept_batch(dp, dq, V, Kd, dd, ds, trials, pos0, dout, h->stream);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(out, dout, sizeof(int) * 2 * trials, cudaMemcpyDeviceToHost, h->stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
+    free_all(h, tmp);
+    CUDA_TRY(e, "spec accept");
+    return SSD_OK;
+}
+
+}  // extern "C"

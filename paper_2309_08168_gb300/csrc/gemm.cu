@@ -1,0 +1,322 @@
+// gemm.cu - skinny projection GEMM of the decode forward (draft, verification
+// and prefill), Y[M x N] = X[M x K] * W^T with W bf16 [N][K], M <= 16.
+//
+// Every projection of the LLaMA-2 decoder (Sec. 4.1) runs through this one
+// kernel: the fused q/k/v projection with RoPE and the KV-cache write, the
+// output and down projections with the residual add, the gate/up projection
+// with SwiGLU, and the lm_head.  The weights are the large operand, so the
+// kernel is "swap-AB": 16 weight rows form the M side of an m16n8k16
+// tensor-core MMA and the <= 16 activation rows form its N side.
+//
+// Batch invariance (needed for greedy self-speculative output to be bit
+// identical to plain autoregressive output, Sec. 1 / App. G.2): the result
+// for activation row m depends only on row m.  The MMA computes every output
+// column independently, the split of K into CTA chunks, into k-interleaved
+// warps and into the fixed-order split-K combine depends on (N, K) only, and
+// every epilogue is element-wise per row.  So a verification row equals the
+// M = 1 forward of the same token at the same position bit for bit.
+//
+// Precision: the fp32 activation rows are split into bf16 hi = rn(x) and
+// lo = rn(x - hi) and both are multiplied (the MMA's N side holds the hi rows
+// then the lo rows), so the product sees ~16 mantissa bits of x; the weights
+// are exact bf16; accumulation is fp32.
+//
+// CTA = 256 threads: warp w handles the 16-row group (w & 3) of the 64-row
+// tile and the k32 blocks b = (w >> 2) (mod 2) of its k-chunk.  The weight
+// chunk (64 rows x kc) is streamed HBM -> shared memory with 16-byte cp.async,
+// then fed to
+// the MMA with a k-permutation: thread (g, t) reads 8 consecutive bf16 of a
+// row, which the A and B fragments both interpret as the same logical k
+// slots, so the product is unchanged and every load is a 128-bit LDS.
+#include "ssd_internal.cuh"
+
+namespace ssd {
+namespace {
+
+__device__ __forceinline__ const bf16* row_src(const GemmArgs& a, int epi, int tile, int r) {
+    const int K = a.K;
+    if (epi == EPI_LOGITS || epi == EPI_RESID) {
+        int n = tile * kTileRows + r;
+        return n < a.N ? a.w0 + (size_t)n * K : nullptr;
+    }
+    if (epi == EPI_SWIGLU) {
+        int i = tile * 32 + (r & 31);
+        if (i >= a.ffn) return nullptr;
+        return (r < 32 ? a.w0 : a.w1) + (size_t)i * K;
+    }
+    // EPI_QKV: q and k tiles hold 32 RoPE pairs (i, i + hd/2) of one head
+    const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
+    const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
+    if (tile < q_tiles + k_tiles) {
+        bool is_q = tile < q_tiles;
+        int tt = is_q ? tile : tile - q_tiles;
+        int head = tt / per_head, j0 = (tt % per_head) * 32;
+        int f = head * hd + (r >> 5) * half + j0 + (r & 31);
+        return (is_q ? a.w0 : a.w1) + (size_t)f * K;
+    }
+    int f = (tile - q_tiles - k_tiles) * kTileRows + r;
+    return a.w2 + (size_t)f * K;
+}
+
+// Splits 8 fp32 activations into bf16 hi = rn(x) and lo = rn(x - hi), so that
+// W * hi + W * lo carries ~16 mantissa bits of x through the bf16 MMA.
+__device__ __forceinline__ void split8(const float4& f0, const float4& f1, uint4& hi, uint4& lo) {
+    const float f[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        __nv_bfloat162 hv = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
+        float2 hf = __bfloat1622float2(hv);
+        __nv_bfloat162 lv = __floats2bfloat162_rn(f[2 * i] - hf.x, f[2 * i + 1] - hf.y);
+        h[i] = *reinterpret_cast<uint32_t*>(&hv);
+        l[i] = *reinterpret_cast<uint32_t*>(&lv);
+    }
+    hi = make_uint4(h[0], h[1], h[2], h[3]);
+    lo = make_uint4(l[0], l[1], l[2], l[3]);
+}
+
+// NPH = n8 tiles per activation half (1: M <= 8, 2: M <= 16).  The MMA's N
+// side holds P = 8*NPH rows of x_hi followed by P rows of x_lo.
+template <int NPH, int EPI>
+__global__ void __launch_bounds__(kGemmThreads) gemm_kernel(const GemmArgs a) {
+    constexpr int NT = 2 * NPH;
+    constexpr int P = 8 * NPH;
+    constexpr int RC = 2 * P;
+    extern __shared__ __align__(16) unsigned char smem[];
+    pdl_launch_dependents();
+    const int tile = blockIdx.x, split = blockIdx.y;
+    const int k0 = split * a.kc;
+    const int kc_eff = min(a.kc, a.K - k0);
+    const int pitch = a.kc * 2 + 64;  // bytes; pitch % 128 == 64 -> conflict-free LDS.128
+    unsigned char* ws = smem;
+    unsigned char* xs = smem + kTileRows * pitch;                // [2P][pitch] hi rows, then lo rows
+    float* red = reinterpret_cast<float*>(xs + 2 * P * pitch);  // [64][RC]
+    float* ys = reinterpret_cast<float*>(smem);                  // [64][16], reuses ws after the MMA
+    __shared__ int s_last;
+
+    // 1. stream the weight chunk (independent of the previous kernel)
+    const int cpr = kc_eff >> 3;  // 16-byte chunks per row
+    for (int c = threadIdx.x; c < kTileRows * cpr; c += kGemmThreads) {
+        int r = c / cpr, cc = c - r * cpr;
+        const bf16* src = row_src(a, EPI, tile, r);
+        const bf16* g = src ? src + k0 + cc * 8 : a.w0;
+        SSD_GUARD(a.err, (((uintptr_t)g & 15u) == 0) && (r * pitch + cc * 16 + 16 <= kTileRows * pitch), 101)
+        cp_async16(ws + r * pitch + cc * 16, g, src ? 16 : 0);
+    }
+    cp_async_commit();
+    // 2. activations of the previous kernel: fp32 -> bf16 hi / lo rows
+    pdl_wait();
+    for (int c = threadIdx.x; c < P * cpr; c += kGemmThreads) {
+        int n = c / cpr, cc = c - n * cpr;
+        uint4 hi = make_uint4(0, 0, 0, 0), lo = make_uint4(0, 0, 0, 0);
+        if (n < a.M) {
+            const float4* src = reinterpret_cast<const float4*>(a.x + (size_t)n * a.K + k0 + cc * 8);
+            split8(__ldcg(src), __ldcg(src + 1), hi, lo);
+        }
+        *reinterpret_cast<uint4*>(xs + n * pitch + cc * 16) = hi;
+        *reinterpret_cast<uint4*>(xs + (P + n) * pitch + cc * 16) = lo;
+    }
+    cp_async_wait<0>();
+    __syncthreads();
+
+    // 3. tensor-core MMA over the chunk
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int rg = warp & 3, kh = warp >> 2;
+    const int g = lane >> 2, tig = lane & 3;
+    float acc[NT][4];
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
+    const unsigned char* ar0 = ws + (rg * 16 + g) * pitch;
+    const unsigned char* ar1 = ar0 + 8 * pitch;
+    const int nb = kc_eff >> 5;
+#pragma unroll 2
+    for (int b = kh; b < nb; b += 2) {
+        const int off = b * 64 + tig * 16;
+        uint4 wa = *reinterpret_cast<const uint4*>(ar0 + off);
+        uint4 wb = *reinterpret_cast<const uint4*>(ar1 + off);
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            uint4 xv = *reinterpret_cast<const uint4*>(xs + (nt * 8 + g) * pitch + off);
+            mma_bf16_16816(acc[nt], wa.x, wb.x, wa.y, wb.y, xv.x, xv.y);
+            mma_bf16_16816(acc[nt], wa.z, wb.z, wa.w, wb.w, xv.z, xv.w);
+        }
+    }
+    if ((kc_eff & 31) && kh == (nb & 1)) {  // k16 tail block
+        const int off = nb * 64 + tig * 8;
+        uint2 wa = *reinterpret_cast<const uint2*>(ar0 + off);
+        uint2 wb = *reinterpret_cast<const uint2*>(ar1 + off);
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            uint2 xv = *reinterpret_cast<const uint2*>(xs + (nt * 8 + g) * pitch + off);
+            mma_bf16_16816(acc[nt], wa.x, wb.x, wa.y, wb.y, xv.x, xv.y);
+        }
+    }
+
+    // 4. fixed-order combines: k-interleave 0 + 1, then x_hi + x_lo -> ys[row][m]
+    const int r0 = rg * 16 + g;
+    if (kh == 1) {
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            int c = nt * 8 + 2 * tig;
+            red[r0 * RC + c] = acc[nt][0];
+            red[r0 * RC + c + 1] = acc[nt][1];
+            red[(r0 + 8) * RC + c] = acc[nt][2];
+            red[(r0 + 8) * RC + c + 1] = acc[nt][3];
+        }
+    }
+    __syncthreads();
+    if (kh == 0) {
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            int c = nt * 8 + 2 * tig;
+            red[r0 * RC + c] = acc[nt][0] + red[r0 * RC + c];
+            red[r0 * RC + c + 1] = acc[nt][1] + red[r0 * RC + c + 1];
+            red[(r0 + 8) * RC + c] = acc[nt][2] + red[(r0 + 8) * RC + c];
+            red[(r0 + 8) * RC + c + 1] = acc[nt][3] + red[(r0 + 8) * RC + c + 1];
+        }
+    }
+    __syncthreads();
+    const int M = a.M;
+    for (int idx = threadIdx.x; idx < kTileRows * M; idx += kGemmThreads) {
+        int m = idx / kTileRows, r = idx - m * kTileRows;
+        ys[r * 16 + m] = red[r * RC + m] + red[r * RC + P + m];
+    }
+    __syncthreads();
+
+    // 5. split-K: the last CTA of the tile sums the partials in split order
+    if (a.ksplit > 1) {
+        const size_t NP = (size_t)a.n_tiles * kTileRows;
+        for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+            int m = idx / kTileRows, r = idx - m * kTileRows;
+            a.partial[((size_t)split * M + m) * NP + (size_t)tile * kTileRows + r] = ys[r * 16 + m];
+        }
+        __threadfence();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            unsigned prev = atomicAdd(&a.counters[tile], 1u);
+            s_last = (prev == (unsigned)(a.ksplit - 1));
+        }
+        __syncthreads();
+        if (!s_last) return;
+        __threadfence();
+        for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+            int m = idx / kTileRows, r = idx - m * kTileRows;
+            const float* p = a.partial + (size_t)m * NP + (size_t)tile * kTileRows + r;
+            float s = __ldcg(p);
+            for (int sp = 1; sp < a.ksplit; ++sp) s += __ldcg(p + (size_t)sp * M * NP);
+            ys[r * 16 + m] = s;
+        }
+        if (threadIdx.x == 0) a.counters[tile] = 0u;
+        __syncthreads();
+    }
+
+    // 6. epilogues (element-wise per activation row)
+    if (EPI == EPI_LOGITS || EPI == EPI_RESID) {
+        for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+            int m = idx / kTileRows, r = idx - m * kTileRows;
+            int n = tile * kTileRows + r;
+            if (n >= a.N) continue;
+            float y = ys[r * 16 + m];
+            float* o = a.out_f32 + (size_t)m * a.ldo + n;
+            if (EPI == EPI_LOGITS) *o = y;
+            else *o = *o + y;
+        }
+    } else if (EPI == EPI_SWIGLU) {
+        for (int idx = threadIdx.x; idx < M * 32; idx += kGemmThreads) {
+            int m = idx >> 5, r = idx & 31;
+            int i = tile * 32 + r;
+            if (i >= a.ffn) continue;
+            float gt = ys[r * 16 + m], up = ys[(r + 32) * 16 + m];
+            a.out_act[(size_t)m * a.ffn + i] = gt / (1.f + expf(-gt)) * up;
+        }
+    } else {  // EPI_QKV
+        const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
+        const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
+        const int pos0 = a.st->pos0;
+        if (tile < q_tiles + k_tiles) {
+            const bool is_q = tile < q_tiles;
+            const int tt = is_q ? tile : tile - q_tiles;
+            const int head = tt / per_head, j0 = (tt % per_head) * 32;
+            for (int idx = threadIdx.x; idx < M * 32; idx += kGemmThreads) {
+                int m = idx >> 5, r = idx & 31;
+                int i = j0 + r, pos = pos0 + m;
+                float x1 = ys[r * 16 + m], x2 = ys[(r + 32) * 16 + m];
+                float2 cs = a.rope[(size_t)pos * half + i];
+                float y1 = x1 * cs.x - x2 * cs.y;
+                float y2 = x2 * cs.x + x1 * cs.y;
+                if (is_q) {
+                    float* q = a.q_out + (size_t)m * a.n_heads * hd + head * hd;
+                    q[i] = y1;
+                    q[i + half] = y2;
+                } else {
+                    f16* k = a.k_cache + ((size_t)head * a.max_seq + pos) * hd;
+                    k[i] = __float2half_rn(y1);
+                    k[i + half] = __float2half_rn(y2);
+                }
+            }
+        } else {
+            const int vt = tile - q_tiles - k_tiles;
+            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+                int m = idx / kTileRows, r = idx - m * kTileRows;
+                int f = vt * kTileRows + r;
+                int head = f / hd, e = f - head * hd;
+                a.v_cache[((size_t)head * a.max_seq + pos0 + m) * hd + e] = __float2half_rn(ys[r * 16 + m]);
+            }
+        }
+    }
+}
+
+template <int NPH, int EPI>
+int launch_one(const GemmArgs& a, cudaStream_t s) {
+    const size_t smem = gemm_smem_bytes(a.kc, a.M);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(a.n_tiles, a.ksplit, 1);
+    cfg.blockDim = dim3(kGemmThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return (int)cudaLaunchKernelEx(&cfg, gemm_kernel<NPH, EPI>, a);
+}
+
+template <int NPH, int EPI>
+int configure_one() {
+    return (int)cudaFuncSetAttribute(gemm_kernel<NPH, EPI>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+}
+
+}  // namespace
+
+int gemm_configure() {
+    int e = 0;
+    e = e ? e : configure_one<1, EPI_LOGITS>();
+    e = e ? e : configure_one<2, EPI_LOGITS>();
+    e = e ? e : configure_one<1, EPI_RESID>();
+    e = e ? e : configure_one<2, EPI_RESID>();
+    e = e ? e : configure_one<1, EPI_SWIGLU>();
+    e = e ? e : configure_one<2, EPI_SWIGLU>();
+    e = e ? e : configure_one<1, EPI_QKV>();
+    e = e ? e : configure_one<2, EPI_QKV>();
+    return e;
+}
+
+size_t gemm_smem_bytes(int kc, int M) {
+    const int P = gemm_half_rows(M);
+    return (size_t)(kTileRows + 2 * P) * (kc * 2 + 64) + (size_t)kTileRows * 2 * P * sizeof(float);
+}
+
+int launch_gemm(int epi, const GemmArgs& a, cudaStream_t s) {
+    const bool two = a.M > 8;
+    switch (epi) {
+        case EPI_LOGITS: return two ? launch_one<2, EPI_LOGITS>(a, s) : launch_one<1, EPI_LOGITS>(a, s);
+        case EPI_RESID: return two ? launch_one<2, EPI_RESID>(a, s) : launch_one<1, EPI_RESID>(a, s);
+        case EPI_SWIGLU: return two ? launch_one<2, EPI_SWIGLU>(a, s) : launch_one<1, EPI_SWIGLU>(a, s);
+        case EPI_QKV: return two ? launch_one<2, EPI_QKV>(a, s) : launch_one<1, EPI_QKV>(a, s);
+    }
+    return (int)cudaErrorInvalidValue;
+}
+
+}  // namespace ssd

@@ -1,0 +1,204 @@
+"""GPU decode path vs the fp64 oracle, through the C ABI.
+
+  * the device input generator writes the same bits as the host generator;
+  * verification (full model) and draft (skip-set model) logits within
+    |d| <= 5e-2 + 1e-2 |oracle| at the tiny config and at layer-truncated
+    LLaMA-2-7B / 70B widths (70B: GQA 64 / 8);
+  * batch invariance: every row of an M-row forward equals, bit for bit, the
+    one-row forward of the same token at the same position (M = 1..16, rows
+    crossing 64-position attention chunks);
+  * greedy self-speculative output is bit-identical to the GPU's own plain
+    autoregressive output (K = 1..15, several skip sets), and the AR tokens
+    agree with the oracle wherever its top-1/top-2 margin exceeds 0.1;
+  * error paths (capacity, state, bad tokens).
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from gpu_util import assert_logits_close, check_tokens_vs_oracle, decoder
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def ssd():
+    import paper_2309_08168_gb300 as m
+    return m
+
+
+@pytest.fixture(scope="module")
+def tiny_setup(ssd):
+    w = synth.workloads()["tiny"]
+    hw = synth.host_weights(w, seed=1)
+    dw = synth.host_to_device_weights(hw)
+    torch.cuda.synchronize()
+    return w, hw, dw
+
+
+def test_device_generator_matches_host(ssd):
+    w = synth.workloads()["tiny"]
+    hw = synth.host_weights(w, seed=5)
+    dw = synth.device_weights(w, seed=5)
+    torch.cuda.synchronize()
+
+    def bits(t):
+        return t.view(torch.int16).cpu().numpy().view(np.uint16)
+
+    assert np.array_equal(bits(dw["embed"]), hw["embed"])
+    assert np.array_equal(bits(dw["lm_head"]), hw["lm_head"])
+    for l in range(w.n_layers):
+        for k in hw["layers"][l]:
+            assert np.array_equal(bits(dw["layers"][l][k]), hw["layers"][l][k]), (l, k)
+    # a slice of a LLaMA-2-7B-sized tensor (scaled skip-set output projection)
+    n = 11008 * 4096
+    t = torch.empty(n, dtype=torch.bfloat16, device="cuda")
+    lib = synth._dev_lib()
+    tid = synth.tensor_id(20, "w_down")
+    lib.synth_fill_bf16_dev(t.data_ptr(), 0, n, 3, tid, synth.scale_const(0.05),
+                            torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    got = bits(t)
+    for first in (0, 12345678, n - 4096):
+        ref = synth.fill_bf16_host(4096, seed=3, tid=tid, scale=0.05, first=first)
+        assert np.array_equal(got[first:first + 4096], ref)
+
+
+def test_tiny_verify_and_draft_logits(ssd, tiny_setup):
+    w, hw, dw = tiny_setup
+    dec = decoder(w, dw, 128)
+    orc = oracle.Oracle(w, hw, max_seq=128)
+    prompt = synth.prompt(w.n_prompt, seed=2, vocab=w.vocab)
+    rows = np.concatenate([prompt[-1:], synth.prompt(w.K, seed=3, vocab=w.vocab)])
+    P = w.n_prompt
+    dec.prefill(prompt)
+    # verification forward over K+1 rows
+    got = dec.debug_forward(False, rows, P - 1)
+    ref = orc.forward_uncached(np.concatenate([prompt[:-1], rows]))[P - 1:]
+    assert_logits_close(got, ref, "verify")
+    # draft steps: the skip-set model, one row at a time, over the prompt's
+    # full-model KV plus its own KV (the cache above was rewritten by the
+    # prefill's positions only; rows >= P-1 are overwritten by the drafts)
+    ref_d = orc.forward_uncached(np.concatenate([prompt[:-1], rows]), n_full=P - 1, mask=w.mask())[P - 1:]
+    for j in range(len(rows)):
+        got_d = dec.debug_forward(True, rows[j:j + 1], P - 1 + j)
+        assert_logits_close(got_d[0], ref_d[j], f"draft {j}")
+    dec.close()
+
+
+@pytest.mark.parametrize("n_rows", [1, 2, 5, 8, 9, 13, 16])
+def test_batch_invariance(ssd, tiny_setup, n_rows):
+    w, hw, dw = tiny_setup
+    dec = decoder(w, dw, 128)
+    prompt = synth.prompt(60, seed=4, vocab=w.vocab)  # rows cross the 64-position chunk
+    rows = synth.prompt(n_rows, seed=10 + n_rows, vocab=w.vocab)
+    dec.prefill(prompt)
+    many = dec.debug_forward(False, rows, 59)
+    one = np.stack([dec.debug_forward(False, rows[r:r + 1], 59 + r)[0] for r in range(n_rows)])
+    assert np.array_equal(many.view(np.uint32), one.view(np.uint32))
+    dec.close()
+
+
+@pytest.mark.parametrize("K", [1, 2, 4, 8, 15])
+def test_tiny_greedy_ssd_equals_ar(ssd, tiny_setup, K):
+    w, hw, dw = tiny_setup
+    dec = decoder(w, dw, 160)
+    prompt = synth.prompt(w.n_prompt, seed=0, vocab=w.vocab)
+    ar, st_ar = dec.generate(prompt, w.n_new, 0)
+    assert st_ar["rounds"] == w.n_new and st_ar["drafted"] == 0
+    for mask in (w.mask(), np.ones(2 * w.n_layers, np.uint8), np.zeros(2 * w.n_layers, np.uint8)):
+        dec.set_skip(mask)
+        sd, st = dec.generate(None, w.n_new, K)
+        assert np.array_equal(ar, sd), (K, mask)
+        assert st["emitted"] == w.n_new == st["rounds"] + st["accepted"]
+        if mask.sum() == 0:
+            assert st["accepted"] == st["drafted"]
+    dec.close()
+
+
+def test_tiny_ar_matches_oracle(ssd, tiny_setup):
+    w, hw, dw = tiny_setup
+    dec = decoder(w, dw, 160)
+    orc = oracle.Oracle(w, hw, max_seq=160)
+    for seed in range(3):
+        prompt = synth.prompt(w.n_prompt, seed=seed, vocab=w.vocab)
+        toks, _ = dec.generate(prompt, w.n_new, 0)
+        n = check_tokens_vs_oracle(toks, orc, prompt, w.n_new)
+        assert n >= 8
+    dec.close()
+
+
+def test_tiny_ssd_stats_and_oracle_rounds(ssd, tiny_setup):
+    """With identical tokens, the acceptance pattern n per round is decided by
+    draft argmaxes; compare the GPU's acceptance with the oracle's run."""
+    w, hw, dw = tiny_setup
+    dec = decoder(w, dw, 160)
+    orc = oracle.Oracle(w, hw, max_seq=160)
+    prompt = synth.prompt(w.n_prompt, seed=0, vocab=w.vocab)
+    toks, st = dec.generate(prompt, w.n_new, w.K)
+    ref, rst = orc.generate(prompt, w.n_new, w.K, mask=w.mask())
+    assert st["drafted"] > 0 and st["accept_rate"] > 0.3
+    if np.array_equal(toks, ref):
+        # tiny margins can flip a draft argmax; totals stay close
+        assert abs(st["accepted"] - rst["accepted"]) <= max(3, rst["accepted"] // 10)
+    dec.close()
+
+
+@pytest.mark.parametrize("shape", ["llama2-7b", "llama2-70b"])
+def test_truncated_big_widths(ssd, shape):
+    """Full-width layers of the big shapes (2 layers; 70B with GQA 64/8)."""
+    w = synth.workloads()[shape].truncated(2, n_prompt=16, n_new=8)
+    hw = synth.host_weights(w, seed=7)
+    dw = synth.host_to_device_weights(hw)
+    torch.cuda.synchronize()
+    dec = decoder(w, dw, 64)
+    orc = oracle.Oracle(w, hw, max_seq=64)
+    prompt = synth.prompt(16, seed=1, vocab=w.vocab)
+    rows = np.concatenate([prompt[-1:], synth.prompt(8, seed=2, vocab=w.vocab)])
+    dec.prefill(prompt)
+    got = dec.debug_forward(False, rows, 15)
+    full = np.concatenate([prompt[:-1], rows])
+    ref = orc.forward_uncached(full)[15:]
+    assert_logits_close(got, ref, f"{shape} verify")
+    got_d = dec.debug_forward(True, rows[:1], 15)
+    ref_d = orc.forward_uncached(full[:16], n_full=15, mask=w.mask())[15]
+    assert_logits_close(got_d[0], ref_d, f"{shape} draft")
+    ar, _ = dec.generate(prompt, 24, 0)
+    sd, st = dec.generate(None, 24, 8)
+    assert np.array_equal(ar, sd)
+    dec.close()
+
+
+def test_errors(ssd, tiny_setup):
+    w, hw, dw = tiny_setup
+    dec = decoder(w, dw, 40)
+    with pytest.raises(ssd.SSDError) as e:
+        dec.generate(None, 4, 2)
+    assert e.value.code == ssd.SSD_ERR_STATE
+    prompt = synth.prompt(32, seed=0, vocab=w.vocab)
+    with pytest.raises(ssd.SSDError) as e:
+        dec.generate(prompt, 9, 2)
+    assert e.value.code == ssd.SSD_ERR_CAPACITY
+    bad = prompt.copy()
+    bad[3] = w.vocab
+    with pytest.raises(ssd.SSDError) as e:
+        dec.prefill(bad)
+    assert e.value.code == ssd.SSD_ERR_INVALID_ARG
+    with pytest.raises(ssd.SSDError) as e:
+        dec.generate(prompt, 4, 16)
+    assert e.value.code == ssd.SSD_ERR_INVALID_ARG
+    with pytest.raises(ssd.SSDError):
+        dec.set_skip(np.ones(3, np.uint8))
+    with pytest.raises(ssd.SSDError):
+        dec.set_sampling(0.0, 0.9)
+    # still usable after errors
+    toks, st = dec.generate(prompt, 8, 2)
+    assert st["emitted"] == 8
+    # prompt of one token: no prefill forward
+    toks1, _ = dec.generate(prompt[:1], 6, 0)
+    toks2, _ = dec.generate(None, 6, 3)
+    assert np.array_equal(toks1, toks2)
+    dec.close()
