@@ -168,6 +168,35 @@ int ssd_debug_spec_accept(ssd_handle* h, const float* p, const float* q, int Kd,
 int ssd_debug_time_forward(ssd_handle* h, int draft, int rows, int gemm_only, int reps,
                            float* ms_per_forward, int* launches, double* weight_bytes);
 
+/* Allocation-free projection.  The paper has no counterpart: this is a
+ * service of this library for callers that cannot allocate device memory
+ * when they need a projection, e.g. a serving process that reserves all of
+ * HBM at start-up and treats any later allocation as an error, a plug-in
+ * whose host framework owns every device allocation, or a latency-critical
+ * loop that must not call cudaMalloc / cudaFree because they can synchronise
+ * the device.  It runs the decoder's projection GEMM kernel alone:
+ *     y[m][n] = sum_k x[m][k] * w[n][k],   m < M, n < N,
+ * w: device bf16 [N][K] row-major; x: device fp32 [M][K] (entering the MMA
+ * as bf16 hi + lo pairs, as inside the decoder); y: device fp32 [M][N]; all
+ * owned by the caller; w and x 16-byte aligned.  1 <= M <= 16, K a positive
+ * multiple of 16.  cuda_stream: the stream to launch on (NULL = legacy
+ * default stream); the call returns after enqueueing the work.
+ * Scratch: nothing is allocated.  The split-K partial sums and the per-tile
+ * arrival counters live in fixed device arrays of the library, 1,048,576
+ * floats and 4,096 counters (about 4 MiB per GPU that loads the library,
+ * held until the process exits).  A problem needs ceil(N/64) <= 4096 tiles
+ * and, when K > 512, ceil(K/512) * M * 64 * ceil(N/64) <= 1,048,576 scratch
+ * floats; larger problems are rejected with SSD_ERR_CAPACITY before any
+ * launch.  The first call on each device does a one-time set-up with that
+ * device current (symbol lookup, kernel attribute, zeroing the counters);
+ * make that first call before any stream capture.  Every call zeroes the
+ * counters it uses on the stream before its kernel; the scratch arrays are
+ * shared by all calls on a device, so calls that overlap on the GPU (other
+ * streams, other threads) race and must be serialised by the caller.
+ * Errors: INVALID_ARG, CAPACITY, CUDA. */
+int ssd_linear_noalloc(const void* w, const float* x, float* y, int N, int K, int M,
+                       void* cuda_stream);
+
 /* Releases everything the handle owns (never the borrowed weights). */
 void ssd_destroy(ssd_handle* h);
 

@@ -28,7 +28,7 @@ SSD_SAMPLE = 1
 # every symbol include/ssd.h declares
 EXPORTS = ("ssd_create", "ssd_set_skip", "ssd_set_sampling", "ssd_prefill", "ssd_generate",
            "ssd_debug_forward", "ssd_debug_spec_accept", "ssd_debug_time_forward", "ssd_destroy",
-           "ssd_last_error")
+           "ssd_last_error", "ssd_linear_noalloc")
 
 
 class ssd_config(ctypes.Structure):
@@ -82,6 +82,8 @@ def _load():
     lib.ssd_debug_spec_accept.argtypes = [H, _VP, _VP, ctypes.c_int, _VP, _VP, ctypes.c_int, ctypes.c_int, _VP]
     lib.ssd_debug_time_forward.argtypes = [H, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                            _VP, _VP, _VP]
+    lib.ssd_linear_noalloc.argtypes = [_VP, _VP, _VP, ctypes.c_int, ctypes.c_int, ctypes.c_int, _VP]
+    lib.ssd_linear_noalloc.restype = ctypes.c_int
     lib.ssd_destroy.argtypes = [H]
     lib.ssd_destroy.restype = None
     lib.ssd_last_error.argtypes = []
@@ -172,6 +174,11 @@ def ssd_debug_time_forward(h: int, draft: bool, rows: int, gemm_only: bool, reps
     _check(lib.ssd_debug_time_forward(h, int(draft), rows, int(gemm_only), reps, ctypes.addressof(ms),
                                       ctypes.addressof(n), ctypes.addressof(b)))
     return ms.value, n.value, b.value
+
+
+def ssd_linear_noalloc(w, x, y, N: int, K: int, M: int, cuda_stream: int | None = None) -> None:
+    """y[M][N] = x[M][K] @ w[N][K]^T on device tensors, without allocating."""
+    _check(lib.ssd_linear_noalloc(_ptr(w), _ptr(x), _ptr(y), N, K, M, cuda_stream))
 
 
 def ssd_destroy(h: int) -> None:

@@ -329,6 +329,11 @@ int check_config(const ssd_config* c) {
 
 }  // namespace
 
+namespace ssd {
+// Records the message that ssd_last_error() returns on this thread.
+int set_last_error(int code, const char* msg) { return fail(code, msg); }
+}  // namespace ssd
+
 extern "C" {
 
 const char* ssd_last_error(void) { return g_err.c_str(); }

@@ -28,6 +28,10 @@
 // the MMA with a k-permutation: thread (g, t) reads 8 consecutive bf16 of a
 // row, which the A and B fragments both interpret as the same logical k
 // slots, so the product is unchanged and every load is a 128-bit LDS.
+#include <mutex>
+#include <string>
+
+#include "ssd.h"
 #include "ssd_internal.cuh"
 
 namespace ssd {
@@ -320,3 +324,112 @@ int launch_gemm(int epi, const GemmArgs& a, cudaStream_t s) {
 }
 
 }  // namespace ssd
+
+// ---------------------------------------------------------------------------
+// ssd_linear_noalloc: the projection GEMM with its split-K scratch in a fixed
+// device array instead of memory the caller or the library allocates.
+//
+// Some callers cannot allocate device memory at the point where they need a
+// projection: a serving process that reserves every byte of HBM at start-up
+// and treats any later allocation as a failure, a plug-in whose host
+// framework owns all device allocations, or a latency-critical loop that
+// must not call cudaMalloc / cudaFree because those calls can synchronise
+// the whole device.  For them this entry point takes device inputs and
+// outputs only and keeps its scratch (split-K partial sums and the per-tile
+// arrival counters) in the static arrays below.  Every GPU that loads the
+// library holds these arrays (about 4 MiB) until the process exits.
+// ---------------------------------------------------------------------------
+namespace ssd {
+namespace {
+
+constexpr size_t kNoAllocPartialFloats = size_t(1) << 20;  // 4 MiB of partial sums
+constexpr int kNoAllocTiles = 4096;                          // 64-row tiles: N <= 262144
+
+static __device__ __align__(256) float g_noalloc_partial[kNoAllocPartialFloats];
+static __device__ __align__(256) unsigned g_noalloc_counters[kNoAllocTiles];
+static __device__ __align__(256) int g_noalloc_err;
+
+// Host-side device addresses of the arrays, resolved once per device.  (In
+// host code the array names are host stand-ins, not device addresses.)
+struct NoAllocDevice {
+    bool ready = false;
+    float* partial = nullptr;
+    unsigned* counters = nullptr;
+    int* err = nullptr;
+};
+constexpr int kNoAllocMaxDevices = 64;
+NoAllocDevice g_noalloc_dev[kNoAllocMaxDevices];
+std::mutex g_noalloc_mu;
+
+int noalloc_setup(int dev, NoAllocDevice** out) {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    NoAllocDevice& d = g_noalloc_dev[dev];
+    if (!d.ready) {
+        cudaError_t e = cudaGetSymbolAddress((void**)&d.partial, g_noalloc_partial);
+        if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&d.counters, g_noalloc_counters);
+        if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&d.err, g_noalloc_err);
+        if (e == cudaSuccess) e = (cudaError_t)configure_one<1, EPI_LOGITS>();
+        if (e == cudaSuccess) e = (cudaError_t)configure_one<2, EPI_LOGITS>();
+        if (e == cudaSuccess) e = cudaMemset(d.counters, 0, sizeof(unsigned) * kNoAllocTiles);
+        if (e != cudaSuccess)
+            return set_last_error(SSD_ERR_CUDA, (std::string("ssd_linear_noalloc set-up: ") +
+                                                 cudaGetErrorString(e)).c_str());
+        d.ready = true;
+    }
+    *out = &d;
+    return SSD_OK;
+}
+
+}  // namespace
+}  // namespace ssd
+
+extern "C" int ssd_linear_noalloc(const void* w, const float* x, float* y, int N, int K, int M,
+                                  void* cuda_stream) {
+    using namespace ssd;
+    if (!w || !x || !y) return set_last_error(SSD_ERR_INVALID_ARG, "ssd_linear_noalloc: NULL pointer");
+    if (((uintptr_t)w & 15u) || ((uintptr_t)x & 15u))
+        return set_last_error(SSD_ERR_INVALID_ARG, "ssd_linear_noalloc: w and x must be 16-byte aligned");
+    if (M < 1 || M > kMaxRows || N < 1 || K < 16 || K % 16)
+        return set_last_error(SSD_ERR_INVALID_ARG,
+                              "ssd_linear_noalloc: need 1 <= M <= 16, N >= 1, K a positive multiple of 16");
+    const int kc = K >= 512 ? 512 : ((K + 63) / 64) * 64;
+    const int ksplit = (K + kc - 1) / kc;
+    const int n_tiles = (N + kTileRows - 1) / kTileRows;
+    const size_t need = ksplit > 1 ? (size_t)ksplit * M * n_tiles * kTileRows : 0;
+    if (n_tiles > kNoAllocTiles || need > kNoAllocPartialFloats)
+        return set_last_error(SSD_ERR_CAPACITY,
+                              ("ssd_linear_noalloc: problem needs " + std::to_string(need) +
+                               " scratch floats and " + std::to_string(n_tiles) +
+                               " tiles; the fixed scratch holds 1048576 floats and 4096 tiles")
+                                  .c_str());
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess || dev < 0 || dev >= kNoAllocMaxDevices)
+        return set_last_error(SSD_ERR_CUDA, "ssd_linear_noalloc: no usable current device");
+    NoAllocDevice* d = nullptr;
+    int rc = noalloc_setup(dev, &d);
+    if (rc) return rc;
+    cudaStream_t s = (cudaStream_t)cuda_stream;
+    // the arrival counters must start at zero (the array keeps the last call's contents)
+    e = cudaMemsetAsync(d->counters, 0, sizeof(unsigned) * n_tiles, s);
+    GemmArgs a{};
+    a.w0 = (const bf16*)w;
+    a.N = N;
+    a.K = K;
+    a.kc = kc;
+    a.ksplit = ksplit;
+    a.n_tiles = n_tiles;
+    a.x = x;
+    a.M = M;
+    a.partial = d->partial;
+    a.counters = d->counters;
+    a.out_f32 = y;
+    a.ldo = N;
+    a.err = d->err;
+    if (e == cudaSuccess)
+        e = (cudaError_t)(M > 8 ? launch_one<2, EPI_LOGITS>(a, s) : launch_one<1, EPI_LOGITS>(a, s));
+    if (e != cudaSuccess)
+        return set_last_error(SSD_ERR_CUDA, (std::string("ssd_linear_noalloc: ") + cudaGetErrorString(e)).c_str());
+    return SSD_OK;
+}
+

@@ -87,6 +87,9 @@ struct AttnArgs {
     int* err;            // device error flag (checked builds)
 };
 
+// sets the thread's ssd_last_error() message and returns code
+int set_last_error(int code, const char* msg);
+
 // launchers (return cudaError_t)
 int gemm_configure();
 int attention_configure();

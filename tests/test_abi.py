@@ -26,7 +26,7 @@ def ssd():
 
 def test_exports_every_declared_symbol(ssd):
     names = _declared()
-    assert len(names) == 10
+    assert len(names) == 11
     assert sorted(ssd.EXPORTS) == names
     lib = ctypes.CDLL(ssd.LIB_PATH)
     for n in names:
@@ -64,6 +64,19 @@ def test_create_rejects_null_weights(ssd):
         ssd.ssd_create(_cfg(ssd), ssd.ssd_weights())
     assert e.value.code == ssd.SSD_ERR_INVALID_ARG
     assert "NULL" in str(e.value)
+
+
+def test_noalloc_rejects_bad_sizes_on_host(ssd):
+    lib = ssd.lib
+    # NULL pointers and sizes are rejected before any device work
+    assert lib.ssd_linear_noalloc(None, None, None, 64, 64, 1, None) == ssd.SSD_ERR_INVALID_ARG
+    buf = (ctypes.c_float * 64)()
+    p = ctypes.addressof(buf) & ~15
+    assert lib.ssd_linear_noalloc(p, p, p, 64, 40, 1, None) == ssd.SSD_ERR_INVALID_ARG  # K % 16
+    assert lib.ssd_linear_noalloc(p, p, p, 64, 64, 17, None) == ssd.SSD_ERR_INVALID_ARG  # M > 16
+    assert lib.ssd_linear_noalloc(p, p, p, 4097 * 64, 64, 1, None) == ssd.SSD_ERR_CAPACITY  # tiles
+    assert lib.ssd_linear_noalloc(p, p, p, 32000, 8192, 16, None) == ssd.SSD_ERR_CAPACITY  # scratch
+    assert "scratch" in ssd.ssd_last_error()
 
 
 def test_null_handle_calls_fail_cleanly(ssd):
