@@ -44,7 +44,7 @@ typedef struct ssd_handle ssd_handle;
 
 /* Model shape (LLaMA-2 decoder, Sec. 4.1 / App. B).
  *   head_dim must be 64 or 128; n_heads a multiple of n_kv_heads (GQA);
- *   d_model a multiple of 64; ffn a multiple of 16; 2 <= vocab <= 32768;
+ *   d_model a multiple of 64; ffn a multiple of 16 and >= 64; 2 <= vocab <= 32768;
  *   max_seq = KV capacity in positions (>= n_prompt + n_new).
  * Numerics: bf16 weights; fp32 residual stream, norms, softmax and
  * accumulation; activations enter each projection as bf16 hi + lo pairs;
@@ -157,16 +157,26 @@ int ssd_debug_spec_accept(ssd_handle* h, const float* p, const float* q, int Kd,
                           int32_t* out);
 
 /* Profiling hook: captures one forward over `rows` rows at the last `rows`
- * positions of the KV cache (full model, or the skip-set model if draft) -
- * or, with gemm_only = 1, only its projection GEMM launches - into a CUDA
- * graph, replays it `reps` times on the handle's stream between two CUDA
- * events, and writes the average time of one replay (ms), the number of
- * kernels in it and the weight bytes one replay streams from HBM.  KV
- * positions [max_seq - rows, max_seq) are overwritten: if they reach into the
- * prefilled prompt, the next ssd_generate needs a prompt again.
+ * positions of the KV cache (full model, or the skip-set model if draft)
+ * into a CUDA graph, replays it `reps` times on the handle's stream between
+ * two CUDA events, and writes the average time of one forward (ms), the
+ * number of kernels in it and the weight bytes it streams from HBM.  With
+ * gemm_only = 1 the time, count and bytes cover the projection ops only
+ * (their share of one replay, read from the forward kernel's device trace).
+ * KV positions [max_seq - rows, max_seq) are overwritten: if they reach into
+ * the prefilled prompt, the next ssd_generate needs a prompt again.
  * 1 <= rows <= 16, reps >= 1.  Errors: INVALID_ARG, CUDA. */
 int ssd_debug_time_forward(ssd_handle* h, int draft, int rows, int gemm_only, int reps,
                            float* ms_per_forward, int* launches, double* weight_bytes);
+
+/* Profiling hook: one forward as in ssd_debug_time_forward, with the device
+ * trace of the forward kernel: op_us[o] = microseconds of op o (from the end
+ * of op o-1 to the end of op o, grid barrier included), op_types[o] = 0
+ * embedding, 1 q/k/v projection, 2 attention, 3 output or down projection,
+ * 4 gate/up projection, 5 lm_head.  max_ops >= 2 + 5 * n_layers is always
+ * enough.  Errors: INVALID_ARG, CUDA. */
+int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, int* op_types,
+                            int max_ops, int* n_ops);
 
 /* Allocation-free projection.  The paper has no counterpart: this is a
  * service of this library for callers that cannot allocate device memory

@@ -28,7 +28,7 @@ SSD_SAMPLE = 1
 # every symbol include/ssd.h declares
 EXPORTS = ("ssd_create", "ssd_set_skip", "ssd_set_sampling", "ssd_prefill", "ssd_generate",
            "ssd_debug_forward", "ssd_debug_spec_accept", "ssd_debug_time_forward", "ssd_destroy",
-           "ssd_last_error", "ssd_linear_noalloc")
+           "ssd_last_error", "ssd_linear_noalloc", "ssd_debug_trace_forward")
 
 
 class ssd_config(ctypes.Structure):
@@ -82,6 +82,8 @@ def _load():
     lib.ssd_debug_spec_accept.argtypes = [H, _VP, _VP, ctypes.c_int, _VP, _VP, ctypes.c_int, ctypes.c_int, _VP]
     lib.ssd_debug_time_forward.argtypes = [H, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                            _VP, _VP, _VP]
+    lib.ssd_debug_trace_forward.argtypes = [H, ctypes.c_int, ctypes.c_int, _VP, _VP, ctypes.c_int, _VP]
+    lib.ssd_debug_trace_forward.restype = ctypes.c_int
     lib.ssd_linear_noalloc.argtypes = [_VP, _VP, _VP, ctypes.c_int, ctypes.c_int, ctypes.c_int, _VP]
     lib.ssd_linear_noalloc.restype = ctypes.c_int
     lib.ssd_destroy.argtypes = [H]
@@ -181,6 +183,21 @@ def ssd_linear_noalloc(w, x, y, N: int, K: int, M: int, cuda_stream: int | None 
     _check(lib.ssd_linear_noalloc(_ptr(w), _ptr(x), _ptr(y), N, K, M, cuda_stream))
 
 
+OP_NAMES = ("embed", "qkv", "attention", "o/down", "gate/up", "lm_head")
+
+
+def ssd_debug_trace_forward(h: int, draft: bool, rows: int):
+    """Returns [(op name, microseconds)] for one forward of the forward kernel."""
+    cfg = config_of(h)
+    cap = 2 + 5 * cfg.n_layers
+    us = np.zeros(cap, dtype=np.float32)
+    ty = np.zeros(cap, dtype=np.int32)
+    n = ctypes.c_int()
+    _check(lib.ssd_debug_trace_forward(h, int(draft), rows, us.ctypes.data, ty.ctypes.data, cap,
+                                       ctypes.addressof(n)))
+    return [(OP_NAMES[ty[i]], float(us[i])) for i in range(n.value)]
+
+
 def ssd_destroy(h: int) -> None:
     if h:
         _configs.pop(h, None)
@@ -264,3 +281,6 @@ class Decoder:
 
     def debug_time_forward(self, draft, rows, gemm_only, reps):
         return ssd_debug_time_forward(self.h, draft, rows, gemm_only, reps)
+
+    def debug_trace_forward(self, draft, rows):
+        return ssd_debug_trace_forward(self.h, draft, rows)

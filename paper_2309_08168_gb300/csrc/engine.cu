@@ -21,6 +21,9 @@
 #include <string>
 #include <vector>
 
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include "ssd.h"
 #include "ssd_internal.cuh"
 
@@ -100,10 +103,22 @@ struct ssd_handle {
     f16* vc = nullptr;
     size_t kv_layer = 0;  // elements per layer of one of K / V
     float* h = nullptr;
-    float* xb = nullptr;  // normalised rows entering a projection [16][d]
+    bf16* xn_hi = nullptr;  // planes of h * g (input of the next normed projection) [16][d]
+    bf16* xn_lo = nullptr;
+    float* ss = nullptr;    // per-64-column sums of h^2 [16][d/64]
     float* q = nullptr;
-    float* attn = nullptr;  // attention output [16][H*hd]
-    float* act = nullptr;   // SwiGLU output [16][ffn]
+    bf16* at_hi = nullptr;  // attention output planes [16][H*hd]
+    bf16* at_lo = nullptr;
+    bf16* ac_hi = nullptr;  // SwiGLU output planes [16][ffn]
+    bf16* ac_lo = nullptr;
+    int n_sms = 0;
+    unsigned* bar = nullptr;            // grid-barrier counter of the forward kernel
+    unsigned long long* trace = nullptr;  // per-op timestamps (profiling hook)
+    CUtensorMap* tmaps = nullptr;       // TMA descriptors (weights, input planes) in device memory
+    int n_tmaps = 0;
+    FwdOp* ops_full = nullptr;          // op lists in device memory
+    FwdOp* ops_draft = nullptr;
+    int n_ops_full = 0, n_ops_draft = 0, max_ops = 0;
     float* logits = nullptr;
     float* p_rows = nullptr;
     float* q_rows = nullptr;
@@ -147,78 +162,223 @@ void drop_graphs(ssd_handle* h, int kind) {
     }
 }
 
-// The forward of one decoder step over M rows: embedding, the sublayers that
-// run (all of them, or those outside the skip set when draft), final norm and
-// lm_head.  Launches only; no host synchronisation (graph-capturable).
-int forward(ssd_handle* h, int M, int src, const int* toks, int pos0, bool draft, bool logits,
-            int* n_launch = nullptr, bool gemm_only = false) {
+// Gains of the RMSNorm in front of the first sublayer that runs after
+// sublayer index s (s = 2l + t, t = 0 attention, 1 MLP), or the final norm.
+const bf16* next_norm(const ssd_handle* h, int s, bool draft) {
+    for (int n = s + 1; n < 2 * h->cfg.n_layers; ++n) {
+        if (draft && h->mask[n]) continue;
+        return (n & 1) ? h->mlp_norm[n >> 1] : h->attn_norm[n >> 1];
+    }
+    return h->final_norm;
+}
+
+// ---------------------------------------------------------------------------
+// TMA descriptors.  Index layout: layer l's wq wk wv wo w_gate w_up w_down at
+// 7l + 0..6, lm_head at 7L, then the input planes: 7L + 1 + (buf * 3 + cls) * 2
+// + plane with buf 0 = normalised rows (K = d), 1 = attention output (K = H*hd),
+// 2 = SwiGLU output (K = ffn); cls = box rows 1 | 8 | 16; plane 0 hi, 1 lo.
+// ---------------------------------------------------------------------------
+int tmap_weight(int l, int which) { return 7 * l + which; }
+int tmap_x(const ssd_handle* h, int buf, int cls, int plane) {
+    return 7 * h->cfg.n_layers + 1 + (buf * 3 + cls) * 2 + plane;
+}
+
+// A 2D bf16 tensor [rows][K] row-major, box 64 (k) x box_rows, 128-byte swizzle,
+// out-of-range elements read as zero.  Checks the TMA rules: 16-byte aligned
+// base, row stride a multiple of 16 bytes, 128-byte inner box.
+int encode_map(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* base, int K, int rows,
+               int box_rows) {
+    if (((uintptr_t)base & 15u) || ((K * 2) % 16) || K < 64 || box_rows < 1 || box_rows > 256)
+        return fail(SSD_ERR_INVALID_ARG, "tensor not suitable for TMA (alignment / row length)");
+    cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+    cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(SSD_ERR_CUDA, "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")");
+    return SSD_OK;
+}
+
+int build_tmaps(ssd_handle* h) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    CUDA_TRY(cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q),
+             "driver entry point");
+    if (!fn || q != cudaDriverEntryPointSuccess) return fail(SSD_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    auto enc = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+    const ssd_config& c = h->cfg;
+    const int L = c.n_layers, d = c.d_model, qd = c.n_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
+    std::vector<CUtensorMap> maps((size_t)h->n_tmaps);
+    int rc = 0;
+    for (int l = 0; l < L && !rc; ++l) {
+        const bf16* w[7] = {h->wq[l], h->wk[l], h->wv[l], h->wo[l], h->w_gate[l], h->w_up[l], h->w_down[l]};
+        const int K[7] = {d, d, d, qd, d, d, c.ffn};
+        const int N[7] = {qd, kvd, kvd, d, c.ffn, c.ffn, d};
+        for (int i = 0; i < 7 && !rc; ++i) rc = encode_map(enc, &maps[tmap_weight(l, i)], w[i], K[i], N[i], 32);
+    }
+    if (!rc) rc = encode_map(enc, &maps[7 * L], h->lm_head, d, c.vocab, 32);
+    const bf16* planes[3][2] = {{h->xn_hi, h->xn_lo}, {h->at_hi, h->at_lo}, {h->ac_hi, h->ac_lo}};
+    const int widths[3] = {d, qd, c.ffn};
+    const int heights[3] = {1, 8, 16};
+    for (int b = 0; b < 3 && !rc; ++b)
+        for (int cls = 0; cls < 3 && !rc; ++cls)
+            for (int pl = 0; pl < 2 && !rc; ++pl)
+                rc = encode_map(enc, &maps[tmap_x(h, b, cls, pl)], planes[b][pl], widths[b], kMaxRows, heights[cls]);
+    if (rc) return rc;
+    CUDA_TRY(cudaMemcpy(h->tmaps, maps.data(), maps.size() * sizeof(CUtensorMap), cudaMemcpyHostToDevice),
+             "tensor map upload");
+    return SSD_OK;
+}
+
+void set_x_maps(const ssd_handle* h, GemmArgs& a, int buf) {
+    for (int cls = 0; cls < 3; ++cls)
+        for (int pl = 0; pl < 2; ++pl) a.tm_x[cls][pl] = h->tmaps + tmap_x(h, buf, cls, pl);
+}
+
+// One projection op: fills the fields every projection shares.
+GemmArgs proj_args(ssd_handle* h, int N, int K, int n_tiles, const bf16* x_hi, const bf16* x_lo) {
+    GemmArgs a{};
+    a.N = N;
+    a.K = K;
+    a.n_tiles = n_tiles;
+    a.n_chunks = (K + kStreamKC - 1) / kStreamKC;
+    a.n_units = n_tiles * a.n_chunks;
+    a.x_hi = x_hi;
+    a.x_lo = x_lo;
+    a.partial = h->partial;
+    a.counters = h->counters;
+    a.st = h->st;
+    a.err = &h->st->err;
+    a.inv_dim = 1.0f / (float)h->cfg.d_model;
+    a.eps = h->cfg.rms_eps;
+    return a;
+}
+
+// The op list of one forward: embedding, the sublayers that run (all of them,
+// or those outside the skip set for the draft model), lm_head last.
+// RMSNorm is folded into the projections: whoever produces the residual
+// stream also writes the bf16 hi / lo planes of h * g_next and per-64-column
+// sums of h^2; the consuming projection scales row m by rsqrt(mean(h^2) + eps).
+std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
     const ssd_config& c = h->cfg;
     const int d = c.d_model, qd = c.n_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
-    cudaStream_t s = h->stream;
-    int launched = 0;
-    const bool aux = !gemm_only;  // norms, embedding, attention
-    if (aux) { LAUNCH(h, launch_embed(h->embed, d, M, src, toks, pos0, h->st, h->h, s), "embed", -1); ++launched; }
+    const int d_tiles = d / kTileRows;
+    std::vector<FwdOp> ops;
+    FwdOp e{};
+    e.type = OP_EMBED;
+    ops.push_back(e);
     for (int l = 0; l < c.n_layers; ++l) {
         const bool run_a = !(draft && h->mask[2 * l]);
         const bool run_m = !(draft && h->mask[2 * l + 1]);
         if (run_a) {
-            if (aux) { LAUNCH(h, launch_rmsnorm(h->h, h->attn_norm[l], d, M, c.rms_eps, h->xb, s), "rmsnorm", l); ++launched; }
-            GemmArgs a{};
+            FwdOp q{};
+            q.type = OP_QKV;
+            GemmArgs& a = q.g;
+            a = proj_args(h, qd + 2 * kvd, d, (qd + 2 * kvd) / kTileRows, h->xn_hi, h->xn_lo);
             a.w0 = h->wq[l]; a.w1 = h->wk[l]; a.w2 = h->wv[l];
-            a.N = qd + 2 * kvd; a.K = d;
-            a.kc = h->p_qkv.kc; a.ksplit = h->p_qkv.ksplit; a.n_tiles = h->p_qkv.n_tiles;
-            a.x = h->xb; a.M = M; a.partial = h->partial; a.counters = h->counters;
+            a.tm_w[0] = h->tmaps + tmap_weight(l, 0);
+            a.tm_w[1] = h->tmaps + tmap_weight(l, 1);
+            a.tm_w[2] = h->tmaps + tmap_weight(l, 2);
+            set_x_maps(h, a, 0);
+            a.ss_in = h->ss; a.ss_in_tiles = d_tiles;
             a.n_heads = c.n_heads; a.n_kv_heads = c.n_kv_heads; a.head_dim = c.head_dim;
             a.max_seq = c.max_seq; a.q_out = h->q;
             a.k_cache = h->kc + (size_t)l * h->kv_layer;
             a.v_cache = h->vc + (size_t)l * h->kv_layer;
-            a.rope = h->rope; a.st = h->st; a.err = &h->st->err;
-            LAUNCH(h, launch_gemm(EPI_QKV, a, s), "qkv projection", l);
-            ++launched;
-            AttnArgs t{};
-            t.q = h->q; t.k_cache = a.k_cache; t.v_cache = a.v_cache; t.out = h->attn;
+            a.rope = h->rope;
+            ops.push_back(q);
+            FwdOp at{};
+            at.type = OP_ATTN;
+            AttnArgs& t = at.at;
+            t.q = h->q; t.k_cache = a.k_cache; t.v_cache = a.v_cache;
+            t.out_hi = h->at_hi; t.out_lo = h->at_lo;
             t.part = h->attn_part; t.counters = h->counters + h->gemm_counters;
-            t.M = M; t.n_heads = c.n_heads; t.n_kv_heads = c.n_kv_heads; t.head_dim = c.head_dim;
+            t.n_heads = c.n_heads; t.n_kv_heads = c.n_kv_heads; t.head_dim = c.head_dim;
             t.max_seq = c.max_seq; t.n_chunks = h->n_chunks;
             t.scale = 1.0f / std::sqrt((float)c.head_dim); t.st = h->st; t.err = &h->st->err;
-            if (aux) { LAUNCH(h, launch_attention(t, s), "attention", l); ++launched; }
-            GemmArgs o{};
-            o.w0 = h->wo[l]; o.N = d; o.K = qd;
-            o.kc = h->p_o.kc; o.ksplit = h->p_o.ksplit; o.n_tiles = h->p_o.n_tiles;
-            o.x = h->attn; o.M = M; o.partial = h->partial; o.counters = h->counters;
-            o.out_f32 = h->h; o.ldo = d; o.st = h->st; o.err = &h->st->err;
-            LAUNCH(h, launch_gemm(EPI_RESID, o, s), "output projection", l);
-            ++launched;
+            ops.push_back(at);
+            FwdOp o{};
+            o.type = OP_RESID;
+            o.g = proj_args(h, d, qd, d_tiles, h->at_hi, h->at_lo);
+            o.g.w0 = h->wo[l];
+            o.g.tm_w[0] = h->tmaps + tmap_weight(l, 3);
+            set_x_maps(h, o.g, 1);
+            o.g.out_f32 = h->h; o.g.ldo = d;
+            o.g.g_next = next_norm(h, 2 * l, draft); o.g.xo_hi = h->xn_hi; o.g.xo_lo = h->xn_lo; o.g.ss_out = h->ss;
+            ops.push_back(o);
         }
         if (run_m) {
-            if (aux) { LAUNCH(h, launch_rmsnorm(h->h, h->mlp_norm[l], d, M, c.rms_eps, h->xb, s), "rmsnorm", l); ++launched; }
-            GemmArgs g{};
-            g.w0 = h->w_gate[l]; g.w1 = h->w_up[l]; g.N = 2 * c.ffn; g.K = d;
-            g.kc = h->p_gu.kc; g.ksplit = h->p_gu.ksplit; g.n_tiles = h->p_gu.n_tiles;
-            g.x = h->xb; g.M = M; g.partial = h->partial; g.counters = h->counters;
-            g.out_act = h->act; g.ffn = c.ffn; g.st = h->st; g.err = &h->st->err;
-            LAUNCH(h, launch_gemm(EPI_SWIGLU, g, s), "gate/up projection", l);
-            ++launched;
-            GemmArgs w{};
-            w.w0 = h->w_down[l]; w.N = d; w.K = c.ffn;
-            w.kc = h->p_down.kc; w.ksplit = h->p_down.ksplit; w.n_tiles = h->p_down.n_tiles;
-            w.x = h->act; w.M = M; w.partial = h->partial; w.counters = h->counters;
-            w.out_f32 = h->h; w.ldo = d; w.st = h->st; w.err = &h->st->err;
-            LAUNCH(h, launch_gemm(EPI_RESID, w, s), "down projection", l);
-            ++launched;
+            FwdOp gu{};
+            gu.type = OP_SWIGLU;
+            gu.g = proj_args(h, 2 * c.ffn, d, (c.ffn + 31) / 32, h->xn_hi, h->xn_lo);
+            gu.g.w0 = h->w_gate[l]; gu.g.w1 = h->w_up[l];
+            gu.g.tm_w[0] = h->tmaps + tmap_weight(l, 4);
+            gu.g.tm_w[1] = h->tmaps + tmap_weight(l, 5);
+            set_x_maps(h, gu.g, 0);
+            gu.g.ss_in = h->ss; gu.g.ss_in_tiles = d_tiles;
+            gu.g.ffn = c.ffn; gu.g.xo_hi = h->ac_hi; gu.g.xo_lo = h->ac_lo;
+            ops.push_back(gu);
+            FwdOp w{};
+            w.type = OP_RESID;
+            w.g = proj_args(h, d, c.ffn, d_tiles, h->ac_hi, h->ac_lo);
+            w.g.w0 = h->w_down[l];
+            w.g.tm_w[0] = h->tmaps + tmap_weight(l, 6);
+            set_x_maps(h, w.g, 2);
+            w.g.out_f32 = h->h; w.g.ldo = d;
+            w.g.g_next = next_norm(h, 2 * l + 1, draft); w.g.xo_hi = h->xn_hi; w.g.xo_lo = h->xn_lo; w.g.ss_out = h->ss;
+            ops.push_back(w);
         }
     }
-    if (logits) {
-        if (aux) { LAUNCH(h, launch_rmsnorm(h->h, h->final_norm, d, M, c.rms_eps, h->xb, s), "final norm", -1); ++launched; }
-        GemmArgs o{};
-        o.w0 = h->lm_head; o.N = c.vocab; o.K = d;
-        o.kc = h->p_head.kc; o.ksplit = h->p_head.ksplit; o.n_tiles = h->p_head.n_tiles;
-        o.x = h->xb; o.M = M; o.partial = h->partial; o.counters = h->counters;
-        o.out_f32 = h->logits; o.ldo = c.vocab; o.st = h->st; o.err = &h->st->err;
-        LAUNCH(h, launch_gemm(EPI_LOGITS, o, s), "lm_head", -1);
-        ++launched;
-    }
-    if (n_launch) *n_launch = launched;
+    FwdOp lg{};
+    lg.type = OP_LOGITS;
+    lg.g = proj_args(h, c.vocab, d, (c.vocab + kTileRows - 1) / kTileRows, h->xn_hi, h->xn_lo);
+    lg.g.w0 = h->lm_head;
+    lg.g.tm_w[0] = h->tmaps + 7 * c.n_layers;
+    set_x_maps(h, lg.g, 0);
+    lg.g.ss_in = h->ss; lg.g.ss_in_tiles = d_tiles;
+    lg.g.out_f32 = h->logits; lg.g.ldo = c.vocab;
+    ops.push_back(lg);
+    return ops;
+}
+
+// (Re)builds the op lists in device memory (outside any stream capture).
+int upload_ops(ssd_handle* h, bool draft) {
+    std::vector<FwdOp> ops = build_ops(h, draft);
+    FwdOp* dst = draft ? h->ops_draft : h->ops_full;
+    CUDA_TRY(cudaMemcpy(dst, ops.data(), ops.size() * sizeof(FwdOp), cudaMemcpyHostToDevice), "op list upload");
+    (draft ? h->n_ops_draft : h->n_ops_full) = (int)ops.size();
+    return SSD_OK;
+}
+
+// One decoder forward over M rows: a single cooperative launch of the forward
+// kernel over the op list (lm_head dropped when no logits are needed).
+// Launches only; no host synchronisation (graph-capturable).
+int forward(ssd_handle* h, int M, int src, const int* toks, int pos0, bool draft, bool logits,
+            int* n_launch = nullptr, unsigned long long* trace = nullptr) {
+    const ssd_config& c = h->cfg;
+    FwdParams p{};
+    p.ops = draft ? h->ops_draft : h->ops_full;
+    p.n_ops = (draft ? h->n_ops_draft : h->n_ops_full) - (logits ? 0 : 1);
+    p.M = M;
+    p.src = src;
+    p.toks = toks;
+    p.pos0_arg = pos0;
+    p.st = h->st;
+    p.embed = h->embed;
+    p.d = c.d_model;
+    p.g0 = next_norm(h, -1, draft);
+    p.h = h->h;
+    p.xn_hi = h->xn_hi;
+    p.xn_lo = h->xn_lo;
+    p.ss = h->ss;
+    p.bar = h->bar;
+    p.err = &h->st->err;
+    p.trace = trace;
+    CUDA_TRY(cudaMemsetAsync(h->bar, 0, sizeof(unsigned), h->stream), "barrier reset");
+    LAUNCH(h, launch_forward(p, c.head_dim, h->n_sms, h->stream), "forward kernel", -1);
+    if (n_launch) *n_launch = 1;
     return SSD_OK;
 }
 
@@ -315,15 +475,15 @@ int check_config(const ssd_config* c) {
         return fail(SSD_ERR_INVALID_ARG, "head_dim must be 64 or 128");
     if (c->n_heads < 1 || c->n_kv_heads < 1 || c->n_heads % c->n_kv_heads)
         return fail(SSD_ERR_INVALID_ARG, "n_heads must be a positive multiple of n_kv_heads");
-    if (c->ffn < 16 || c->ffn % 16) return fail(SSD_ERR_INVALID_ARG, "ffn must be a positive multiple of 16");
+    if (c->ffn < 64 || c->ffn % 16) return fail(SSD_ERR_INVALID_ARG, "ffn must be a multiple of 16, at least 64");
     if (c->vocab < 2 || c->vocab > 32768) return fail(SSD_ERR_INVALID_ARG, "vocab must be in [2, 32768]");
     if (c->max_seq < 2 || c->max_seq > (1 << 24)) return fail(SSD_ERR_INVALID_ARG, "max_seq out of range");
     if (!(c->rms_eps > 0.f) || !(c->rope_theta > 0.f))
         return fail(SSD_ERR_INVALID_ARG, "rms_eps and rope_theta must be positive");
     const int G = c->n_heads / c->n_kv_heads;
-    size_t attn_smem = 2 * kAttnChunk * (c->head_dim * 2 + 16) + (size_t)G * kMaxRows * c->head_dim * 4 +
-                       8 * kAttnChunk * 4;
-    if (attn_smem > 200 * 1024) return fail(SSD_ERR_INVALID_ARG, "n_heads / n_kv_heads too large");
+    if (attention_smem_bytes(c->head_dim, G, 8) > forward_smem_bytes(8) ||
+        attention_smem_bytes(c->head_dim, G, kMaxRows) > forward_smem_bytes(kMaxRows))
+        return fail(SSD_ERR_INVALID_ARG, "n_heads / n_kv_heads too large");
     return SSD_OK;
 }
 
@@ -384,8 +544,9 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
         h->own_stream = true;
     }
     {
-        int e1 = gemm_configure(), e2 = attention_configure(), e3 = sampling_configure();
+        int e1 = forward_configure(), e2 = gemm_configure(), e3 = sampling_configure();
         int e = e1 ? e1 : (e2 ? e2 : e3);
+        if (!e) e = (int)cudaDeviceGetAttribute(&h->n_sms, cudaDevAttrMultiProcessorCount, h->device);
         if (e) return bail(fail(SSD_ERR_CUDA, std::string("kernel setup: ") + cudaGetErrorString((cudaError_t)e)));
     }
 
@@ -430,7 +591,9 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
     size_t part = 0;
     int tiles = 0;
     for (const GemmPlan* p : {&h->p_qkv, &h->p_o, &h->p_gu, &h->p_down, &h->p_head}) {
-        part = std::max(part, (size_t)p->ksplit * kMaxRows * p->n_tiles * kTileRows);
+        const int K = p == &h->p_o ? qd : (p == &h->p_down ? c.ffn : d);
+        const size_t chunks = (size_t)(K + kStreamKC - 1) / kStreamKC;
+        part = std::max(part, chunks * kMaxRows * p->n_tiles * kTileRows);
         tiles = std::max(tiles, p->n_tiles);
     }
     h->gemm_counters = tiles;
@@ -442,9 +605,12 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
     h->kv_layer = (size_t)c.n_kv_heads * c.max_seq * c.head_dim;
     const size_t HD = c.head_dim;
     if ((rc = dalloc(h, &h->kc, h->kv_layer * L, &B)) || (rc = dalloc(h, &h->vc, h->kv_layer * L, &B)) ||
-        (rc = dalloc(h, &h->h, (size_t)kMaxRows * d, &B)) || (rc = dalloc(h, &h->xb, (size_t)kMaxRows * d, &B)) ||
-        (rc = dalloc(h, &h->q, (size_t)kMaxRows * qd, &B)) || (rc = dalloc(h, &h->attn, (size_t)kMaxRows * qd, &B)) ||
-        (rc = dalloc(h, &h->act, (size_t)kMaxRows * F, &B)) ||
+        (rc = dalloc(h, &h->h, (size_t)kMaxRows * d, &B)) ||
+        (rc = dalloc(h, &h->xn_hi, (size_t)kMaxRows * d, &B)) || (rc = dalloc(h, &h->xn_lo, (size_t)kMaxRows * d, &B)) ||
+        (rc = dalloc(h, &h->ss, (size_t)kMaxRows * (d / kTileRows), &B)) ||
+        (rc = dalloc(h, &h->q, (size_t)kMaxRows * qd, &B)) ||
+        (rc = dalloc(h, &h->at_hi, (size_t)kMaxRows * qd, &B)) || (rc = dalloc(h, &h->at_lo, (size_t)kMaxRows * qd, &B)) ||
+        (rc = dalloc(h, &h->ac_hi, (size_t)kMaxRows * F, &B)) || (rc = dalloc(h, &h->ac_lo, (size_t)kMaxRows * F, &B)) ||
         (rc = dalloc(h, &h->logits, (size_t)kMaxRows * V, &B)) ||
         (rc = dalloc(h, &h->p_rows, (size_t)kMaxRows * V, &B)) ||
         (rc = dalloc(h, &h->q_rows, (size_t)kMaxRows * V, &B)) || (rc = dalloc(h, &h->partial, part, &B)) ||
@@ -453,7 +619,14 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
         (rc = dalloc(h, &h->rope, (size_t)c.max_seq * (HD / 2), &B)) ||
         (rc = dalloc(h, &h->tok, (size_t)c.max_seq + kMaxRows, &B)) ||
         (rc = dalloc(h, &h->out, (size_t)c.max_seq, &B)) || (rc = dalloc(h, &h->argbuf, 32, &B)) ||
-        (rc = dalloc(h, &h->st, 1, &B)))
+        (rc = dalloc(h, &h->st, 1, &B)) || (rc = dalloc(h, &h->bar, 4, &B)))
+        return bail(rc);
+    h->max_ops = 2 + 5 * L;
+    h->n_tmaps = 7 * L + 1 + 18;
+    if ((rc = dalloc(h, &h->tmaps, (size_t)h->n_tmaps, &B)) ||
+        (rc = dalloc(h, &h->ops_full, (size_t)h->max_ops, &B)) ||
+        (rc = dalloc(h, &h->ops_draft, (size_t)h->max_ops, &B)) ||
+        (rc = dalloc(h, &h->trace, (size_t)h->max_ops + 1, &B)))
         return bail(rc);
     {
         cudaError_t e = cudaMallocHost(&h->st_host, sizeof(DecodeState));
@@ -477,6 +650,7 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
     if (e == cudaSuccess) e = cudaMemsetAsync(h->vc, 0, h->kv_layer * L * sizeof(f16), h->stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
     if (e != cudaSuccess) return bail(fail(SSD_ERR_CUDA, std::string("init: ") + cudaGetErrorString(e)));
+    if ((rc = build_tmaps(h)) || (rc = upload_ops(h, false)) || (rc = upload_ops(h, true))) return bail(rc);
     *out = h;
     return SSD_OK;
 }
@@ -486,9 +660,11 @@ int ssd_set_skip(ssd_handle* h, const uint8_t* mask, int n_sublayers) {
     if (n_sublayers != 2 * h->cfg.n_layers) return fail(SSD_ERR_INVALID_ARG, "n_sublayers must be 2 * n_layers");
     for (int i = 0; i < n_sublayers; ++i)
         if (mask[i] > 1) return fail(SSD_ERR_INVALID_ARG, "mask values must be 0 or 1");
+    CUDA_TRY(cudaSetDevice(h->device), "set device");
+    CUDA_TRY(cudaStreamSynchronize(h->stream), "sync");
     h->mask.assign(mask, mask + n_sublayers);
     drop_graphs(h, G_DRAFT);
-    return SSD_OK;
+    return upload_ops(h, true);
 }
 
 int ssd_set_sampling(ssd_handle* h, float temperature, float top_p) {
@@ -508,6 +684,7 @@ int ssd_prefill(ssd_handle* h, const int32_t* prompt, int n_prompt) {
         if (prompt[i] < 0 || prompt[i] >= h->cfg.vocab) return fail(SSD_ERR_INVALID_ARG, "prompt token out of range");
     CUDA_TRY(cudaSetDevice(h->device), "set device");
     h->prefilled = false;
+    CUDA_TRY(cudaMemsetAsync(&h->st->err, 0, sizeof(int), h->stream), "error flag reset");
     if (n_prompt > 1)
         CUDA_TRY(cudaMemcpyAsync(h->tok, prompt, sizeof(int) * (n_prompt - 1), cudaMemcpyHostToDevice, h->stream),
                  "prompt upload");
@@ -517,6 +694,11 @@ int ssd_prefill(ssd_handle* h, const int32_t* prompt, int n_prompt) {
         if (rc) return rc;
     }
     CUDA_TRY(cudaStreamSynchronize(h->stream), "prefill");
+    {
+        int derr = 0;
+        CUDA_TRY(cudaMemcpy(&derr, &h->st->err, sizeof(int), cudaMemcpyDeviceToHost), "error flag");
+        if (derr == kDevErrTimeout) return fail(SSD_ERR_TIMEOUT, "a grid barrier of the forward kernel timed out");
+    }
 #ifdef SSD_CHECKED
     {
         int derr = 0;
@@ -588,7 +770,11 @@ int ssd_generate(ssd_handle* h, const int32_t* prompt, int n_prompt, int n_new, 
         CUDA_TRY(cudaEventRecord(ev[2], h->stream), "event");
         CUDA_TRY(cudaMemcpyAsync(h->emitted_host, &h->st->emitted, sizeof(int), cudaMemcpyDeviceToHost, h->stream),
                  "state read");
+        CUDA_TRY(cudaMemcpyAsync(h->emitted_host + 1, &h->st->err, sizeof(int), cudaMemcpyDeviceToHost, h->stream),
+                 "state read");
         CUDA_TRY(cudaStreamSynchronize(h->stream), "round");
+        if (h->emitted_host[1] == kDevErrTimeout)
+            return fail(SSD_ERR_TIMEOUT, "a grid barrier of the forward kernel timed out");
         const int e = *h->emitted_host;
         if (e <= emitted || e > n_new) return fail(SSD_ERR_CUDA, "decode state corrupted");
         emitted = e;
@@ -641,32 +827,51 @@ int ssd_debug_forward(ssd_handle* h, int draft, const int32_t* tokens, int n_row
     return SSD_OK;
 }
 
+// Per-op durations (us) of one forward replay from the device trace.
+int trace_forward(ssd_handle* h, cudaGraphExec_t exec, int n_ops, std::vector<float>* us) {
+    std::vector<unsigned long long> t((size_t)n_ops + 1);
+    CUDA_TRY(cudaGraphLaunch(exec, h->stream), "traced replay");
+    CUDA_TRY(cudaMemcpyAsync(t.data(), h->trace, t.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost,
+                             h->stream), "trace read");
+    CUDA_TRY(cudaStreamSynchronize(h->stream), "trace");
+    us->resize(n_ops);
+    for (int o = 0; o < n_ops; ++o) (*us)[o] = (float)((double)(t[o + 1] - t[o]) * 1e-3);
+    return SSD_OK;
+}
+
+int capture_debug_forward(ssd_handle* h, int draft, int rows, bool traced, cudaGraphExec_t* exec, int* n) {
+    const int pos0 = h->cfg.max_seq - rows;
+    int* dt = h->tok + h->cfg.max_seq;
+    CUDA_TRY(cudaMemsetAsync(dt, 0, sizeof(int) * rows, h->stream), "tokens");
+    cudaGraph_t g = nullptr;
+    CUDA_TRY(cudaStreamBeginCapture(h->stream, cudaStreamCaptureModeThreadLocal), "begin capture");
+    int rc = forward(h, rows, SRC_TOKENS, dt, pos0, draft != 0, true, n, traced ? h->trace : nullptr);
+    cudaError_t e = cudaStreamEndCapture(h->stream, &g);
+    if (rc) { if (g) cudaGraphDestroy(g); return rc; }
+    CUDA_TRY(e, "end capture");
+    e = cudaGraphInstantiate(exec, g, 0);
+    cudaGraphDestroy(g);
+    CUDA_TRY(e, "graph instantiate");
+    if (pos0 < h->n_prompt) h->prefilled = false;  // the prompt's KV is overwritten
+    return SSD_OK;
+}
+
 int ssd_debug_time_forward(ssd_handle* h, int draft, int rows, int gemm_only, int reps, float* ms_per_forward,
                            int* launches, double* weight_bytes) {
     if (!h || !ms_per_forward || !launches || !weight_bytes) return fail(SSD_ERR_INVALID_ARG, "NULL argument");
     if (rows < 1 || rows > kMaxRows || reps < 1 || rows > h->cfg.max_seq)
         return fail(SSD_ERR_INVALID_ARG, "rows in [1, 16] and reps >= 1 required");
     CUDA_TRY(cudaSetDevice(h->device), "set device");
-    const int pos0 = h->cfg.max_seq - rows;
-    int* dt = h->tok + h->cfg.max_seq;
-    CUDA_TRY(cudaMemsetAsync(dt, 0, sizeof(int) * rows, h->stream), "tokens");
-    DecodeState* init = h->st_host;
-    std::memset(init, 0, sizeof(DecodeState));
-    init->pos0 = pos0;
-    CUDA_TRY(cudaMemcpyAsync(h->st, init, sizeof(DecodeState), cudaMemcpyHostToDevice, h->stream), "state");
-    cudaGraph_t g = nullptr;
+    cudaGraphExec_t exec = nullptr, traced = nullptr;
     int n = 0;
-    CUDA_TRY(cudaStreamBeginCapture(h->stream, cudaStreamCaptureModeThreadLocal), "begin capture");
-    int rc = forward(h, rows, SRC_TOKENS, dt, pos0, draft != 0, true, &n, gemm_only != 0);
-    cudaError_t e = cudaStreamEndCapture(h->stream, &g);
-    if (rc) { if (g) cudaGraphDestroy(g); return rc; }
-    CUDA_TRY(e, "end capture");
-    cudaGraphExec_t exec = nullptr;
-    e = cudaGraphInstantiate(&exec, g, 0);
-    cudaGraphDestroy(g);
-    CUDA_TRY(e, "graph instantiate");
+    int rc = capture_debug_forward(h, draft, rows, false, &exec, &n);
+    if (!rc && gemm_only) rc = capture_debug_forward(h, draft, rows, true, &traced, &n);
+    if (rc) {
+        if (exec) cudaGraphExecDestroy(exec);
+        return rc;
+    }
     cudaEvent_t e0 = nullptr, e1 = nullptr;
-    e = cudaEventCreate(&e0);
+    cudaError_t e = cudaEventCreate(&e0);
     if (e == cudaSuccess) e = cudaEventCreate(&e1);
     if (e == cudaSuccess) e = cudaGraphLaunch(exec, h->stream);  // warm-up
     if (e == cudaSuccess) e = cudaEventRecord(e0, h->stream);
@@ -678,11 +883,57 @@ int ssd_debug_time_forward(ssd_handle* h, int draft, int rows, int gemm_only, in
     if (e0) cudaEventDestroy(e0);
     if (e1) cudaEventDestroy(e1);
     cudaGraphExecDestroy(exec);
-    CUDA_TRY(e, "timing");
-    *ms_per_forward = ms / reps;
+    if (e != cudaSuccess) {
+        if (traced) cudaGraphExecDestroy(traced);
+        CUDA_TRY(e, "timing");
+    }
+    ms /= reps;
     *launches = n;
-    *weight_bytes = forward_weight_bytes(h, draft != 0, gemm_only != 0);
-    if (pos0 < h->n_prompt) h->prefilled = false;  // the prompt's KV was overwritten
+    *weight_bytes = forward_weight_bytes(h, draft != 0, false);
+    if (gemm_only) {
+        // share of the projection ops in one traced replay, applied to the event-timed forward
+        std::vector<float> us;
+        const int n_ops = draft ? h->n_ops_draft : h->n_ops_full;
+        rc = trace_forward(h, traced, n_ops, &us);
+        cudaGraphExecDestroy(traced);
+        if (rc) return rc;
+        std::vector<FwdOp> ops = build_ops(h, draft != 0);
+        double all = 0.0, proj = 0.0;
+        int n_proj = 0;
+        for (int o = 0; o < n_ops; ++o) {
+            all += us[o];
+            if (ops[o].type != OP_EMBED && ops[o].type != OP_ATTN) { proj += us[o]; ++n_proj; }
+        }
+        ms = (float)(ms * (all > 0 ? proj / all : 1.0));
+        *launches = n_proj;
+        *weight_bytes = forward_weight_bytes(h, draft != 0, true);
+    }
+    *ms_per_forward = ms;
+    return SSD_OK;
+}
+
+int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, int* op_types, int max_ops,
+                            int* n_ops_out) {
+    if (!h || !op_us || !op_types || !n_ops_out) return fail(SSD_ERR_INVALID_ARG, "NULL argument");
+    if (rows < 1 || rows > kMaxRows || rows > h->cfg.max_seq) return fail(SSD_ERR_INVALID_ARG, "rows in [1, 16]");
+    const int n_ops = draft ? h->n_ops_draft : h->n_ops_full;
+    if (max_ops < n_ops) return fail(SSD_ERR_INVALID_ARG, "max_ops smaller than the op list");
+    CUDA_TRY(cudaSetDevice(h->device), "set device");
+    cudaGraphExec_t traced = nullptr;
+    int n = 0;
+    int rc = capture_debug_forward(h, draft, rows, true, &traced, &n);
+    if (rc) return rc;
+    std::vector<float> us;
+    CUDA_TRY(cudaGraphLaunch(traced, h->stream), "warm-up");
+    rc = trace_forward(h, traced, n_ops, &us);
+    cudaGraphExecDestroy(traced);
+    if (rc) return rc;
+    std::vector<FwdOp> ops = build_ops(h, draft != 0);
+    for (int o = 0; o < n_ops; ++o) {
+        op_us[o] = us[o];
+        op_types[o] = ops[o].type;
+    }
+    *n_ops_out = n_ops;
     return SSD_OK;
 }
 

@@ -1,0 +1,849 @@
+// forward_kernel.cu - one decoder forward (draft step, verification, prefill
+// chunk) as a single persistent, cooperative kernel.
+//
+// Batch-1 decoding streams every weight byte once per forward and is bound by
+// HBM (Sec. 3.1).  At LLaMA-2 7B scale a projection takes 5-30 us at full
+// bandwidth, so per-kernel ramp-up and drain would cost a large fraction of
+// the step.  Instead one CTA per SM walks the forward's op list
+//     embed -> [QKV -> attention -> O] -> [gate/up -> down] -> ... -> lm_head
+// (sublayers in the skip set z are simply absent from the draft's list,
+// Sec. 3.2 / 3.3) with a grid barrier between dependent ops.  Before entering
+// a barrier every CTA already requests the weights of its first units of the
+// next projection (they do not depend on the previous op), so the barrier's
+// latency overlaps HBM streaming.  Every wait is bounded: a barrier that does
+// not complete within ~2 s records an error code and the CTAs return.
+//
+// Projections (all of them: q/k/v + RoPE + KV write, output and down with the
+// residual add, gate/up with SwiGLU, lm_head): swap-AB tensor-core MMA,
+// mma.sync m16n8k16 bf16 -> fp32, 16 weight rows on the MMA's M side, the
+// activation rows as bf16 hi + lo planes on its N side (~16 mantissa bits).
+// Work unit = 64-row tile x 256-wide k chunk (32 KB of weights); each CTA
+// owns an equal contiguous range of units in tile-major order, streamed
+// through a 4-stage cp.async ring; a tile split over several CTAs is summed
+// in segment order by the CTA that finishes it last (arrival counter, no
+// waiting).  RMSNorm is folded in: the producer of the residual stream writes
+// the planes of h * g_next and per-64-column sums of h^2, the consumer scales
+// row m by rsqrt(mean(h^2) + eps) in its epilogue (W (h g r) = r W (h g)).
+//
+// Attention: units = (KV head, absolute 64-position chunk); the partial
+// softmax of a row over a chunk depends only on the row and the chunk, and
+// the CTA that completes a head last combines its chunks in chunk order.
+//
+// Coherence: L1 is not coherent across SMs within one launch, so every load of
+// data another CTA wrote during this launch goes through L2 (cp.async.cg,
+// ld.global.cg); stores are write-through.
+//
+// Batch invariance (greedy self-speculative output must equal autoregressive
+// output bit for bit, Sec. 1 / App. G.2): row m's result depends only on row
+// m - MMA columns are independent, unit partitions and combine orders depend
+// on the shapes and the grid only, epilogues are per row, attention chunks are
+// absolute positions.
+#include "ssd_internal.cuh"
+
+namespace ssd {
+namespace {
+
+constexpr int KC = kStreamKC;
+constexpr int S = kStreamStages;
+constexpr int ROWB = KC * 2;  // bytes of one 64-row tile row of a unit
+constexpr unsigned long long kBarrierTimeoutNs = 2000000000ull;
+// 8 consumer warps (MMA, epilogues, attention, embedding) + 1 producer warp (TMA)
+constexpr int kConsumers = 256;
+constexpr int kFwdThreads = kConsumers + 32;
+
+// barrier among the consumer warps only (the producer keeps streaming)
+__device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
+
+
+__device__ __forceinline__ unsigned long long globaltimer() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Grid-wide barrier for a cooperative launch (all CTAs co-resident).  The
+// counter only grows during a launch; `target` = gridDim.x * (barrier index).
+// Returns false (and records SSD_DEV_ERR_TIMEOUT) if the others do not arrive
+// within kBarrierTimeoutNs, or if another CTA already gave up.
+__device__ bool grid_barrier(unsigned* bar, unsigned target, int* err) {
+    __shared__ int s_ok;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        atomicAdd(bar, 1u);
+        int ok = 1;
+        const unsigned long long t0 = globaltimer();
+        while (ld_acquire(bar) < target) {
+            if (*(volatile int*)err) { ok = 0; break; }
+            if (globaltimer() - t0 > kBarrierTimeoutNs) {
+                atomicCAS(err, 0, kDevErrTimeout);
+                ok = 0;
+                break;
+            }
+            __nanosleep(32);
+        }
+        __threadfence();
+        s_ok = ok;
+    }
+    __syncthreads();
+    return s_ok != 0;
+}
+
+__device__ __forceinline__ int unit_owner(long long u, long long U, long long G) {
+    return (int)(((u + 1) * G + U - 1) / U - 1);
+}
+
+// An op's units are split over the first min(U, grid) CTAs, so every CTA that
+// takes part owns at least one unit and the owners of consecutive units are
+// consecutive CTAs (the segment arithmetic of the projection op relies on it).
+__device__ __forceinline__ long long op_ctas(long long U) { return U < gridDim.x ? U : (long long)gridDim.x; }
+
+__device__ __forceinline__ void my_units(long long U, int* u_begin, int* n_my) {
+    const long long G = op_ctas(U), b = blockIdx.x;
+    if (b >= G) { *u_begin = 0; *n_my = 0; return; }
+    *u_begin = (int)(b * U / G);
+    *n_my = (int)((b + 1) * U / G) - *u_begin;
+}
+
+__device__ __forceinline__ bool is_gemm(int type) { return type >= OP_QKV && type <= OP_LOGITS && type != OP_ATTN; }
+
+__device__ __forceinline__ int epi_of(int type) {
+    return type == OP_QKV ? EPI_QKV : type == OP_RESID ? EPI_RESID : type == OP_SWIGLU ? EPI_SWIGLU : EPI_LOGITS;
+}
+
+// ---------------------------------------------------------------------------
+// TMA + mbarrier helpers
+// ---------------------------------------------------------------------------
+constexpr unsigned long long kWaitTimeoutNs = 2000000000ull;
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, unsigned count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+// adds expected bytes without arriving (the weights of a unit, requested early)
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, unsigned bytes) {
+    asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+// plain arrival (a consumer warp releasing a stage)
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+// arrives (count 1) and adds expected bytes (the activations of the unit)
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, unsigned bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, unsigned parity) {
+    unsigned ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// bounded wait: false (error recorded) after kWaitTimeoutNs
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity, int* err) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = globaltimer();
+    while (!mbar_try_wait(bar, parity)) {
+        if (globaltimer() - t0 > kWaitTimeoutNs) {
+            atomicCAS(err, 0, kDevErrTimeout);
+            return false;
+        }
+    }
+    return true;
+}
+// 2D tiled TMA load of one box into shared memory, completing on `bar`.  x is
+// the innermost (k) coordinate; every x used here is a multiple of 64
+// elements (128 bytes), so the 16-byte rule for x * element size holds.
+__device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, int x, int y, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+        ::"r"(smem_u32(dst)), "l"(tmap), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// projection op
+// ---------------------------------------------------------------------------
+// Stage layout (every box 1 KB aligned, 128-byte swizzle: 16-byte chunk c of
+// row r sits at chunk c ^ (r & 7)):
+//   weights: 4 k-boxes x 64 rows x 128 B  (k-box stride 8 KB; rows 0-31 and
+//            32-63 are two TMA boxes of 4 KB)
+//   inputs : 4 k-boxes x (P hi rows + P lo rows) x 128 B
+template <int P>
+struct GemmSmem {
+    static constexpr int WB = kTileRows * ROWB;         // 32 KB
+    static constexpr int XKB = 2 * P * 128;             // input bytes per k-box
+    static constexpr int XB = 4 * XKB;
+    static constexpr int STAGE = WB + XB;
+    static constexpr int RC = 2 * P;
+    static constexpr size_t BYTES = 1024 + (size_t)S * STAGE + kTileRows * RC * 4 + kTileRows * 16 * 4;
+};
+
+__device__ __forceinline__ int x_class(int M) { return M == 1 ? 0 : (M <= 8 ? 1 : 2); }
+__device__ __forceinline__ int x_rows(int M) { return M == 1 ? 1 : (M <= 8 ? 8 : 16); }
+
+// the two 32-row TMA boxes of a 64-row tile: (map, first row) for rows 0-31 and 32-63
+__device__ __forceinline__ void tile_boxes(const GemmArgs& a, int epi, int tile, const void** m0, int* r0,
+                                           const void** m1, int* r1) {
+    if (epi == EPI_LOGITS || epi == EPI_RESID) {
+        *m0 = *m1 = a.tm_w[0];
+        *r0 = tile * kTileRows;
+        *r1 = *r0 + 32;
+    } else if (epi == EPI_SWIGLU) {  // gate rows, up rows
+        *m0 = a.tm_w[0];
+        *m1 = a.tm_w[1];
+        *r0 = *r1 = tile * 32;
+    } else {  // QKV: q / k tiles hold RoPE pairs (i, i + hd/2); v tiles are plain
+        const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
+        const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
+        if (tile < q_tiles + k_tiles) {
+            const bool is_q = tile < q_tiles;
+            const int tt = is_q ? tile : tile - q_tiles;
+            const int head = tt / per_head, j0 = (tt % per_head) * 32;
+            *m0 = *m1 = is_q ? a.tm_w[0] : a.tm_w[1];
+            *r0 = head * hd + j0;
+            *r1 = head * hd + half + j0;
+        } else {
+            *m0 = *m1 = a.tm_w[2];
+            *r0 = (tile - q_tiles - k_tiles) * kTileRows;
+            *r1 = *r0 + 32;
+        }
+    }
+}
+
+__device__ __forceinline__ int unit_kboxes(const GemmArgs& a, int u) {
+    const int k0 = (u % a.n_chunks) * KC;
+    return min(4, (a.K - k0 + 63) / 64);
+}
+
+// weights of unit u into a stage (one thread): expect_tx without arriving
+template <int P>
+__device__ __forceinline__ void tma_weights(const GemmArgs& a, int epi, int u, unsigned char* st, uint64_t* bar) {
+    const int tile = u / a.n_chunks, k0 = (u - tile * a.n_chunks) * KC;
+    const int nkb = unit_kboxes(a, u);
+    const void *m0, *m1;
+    int r0, r1;
+    tile_boxes(a, epi, tile, &m0, &r0, &m1, &r1);
+    mbar_expect_tx(bar, (unsigned)nkb * 2u * 32u * 128u);
+    for (int kb = 0; kb < nkb; ++kb) {
+        tma_load_2d(st + kb * 8192, m0, k0 + kb * 64, r0, bar);
+        tma_load_2d(st + kb * 8192 + 4096, m1, k0 + kb * 64, r1, bar);
+    }
+}
+
+// input planes of unit u into a stage (one thread): arrive + expect_tx
+template <int P>
+__device__ __forceinline__ void tma_inputs(const GemmArgs& a, int M, int u, unsigned char* st, uint64_t* bar) {
+    using L = GemmSmem<P>;
+    const int k0 = (u % a.n_chunks) * KC;
+    const int nkb = unit_kboxes(a, u);
+    const int cls = x_class(M), rows = x_rows(M);
+    mbar_arrive_expect_tx(bar, (unsigned)nkb * 2u * (unsigned)rows * 128u);
+    unsigned char* xs = st + L::WB;
+    for (int kb = 0; kb < nkb; ++kb) {
+        tma_load_2d(xs + kb * L::XKB, a.tm_x[cls][0], k0 + kb * 64, 0, bar);
+        tma_load_2d(xs + kb * L::XKB + P * 128, a.tm_x[cls][1], k0 + kb * 64, 0, bar);
+    }
+}
+
+// Pipeline state of the CTA, carried across ops.  Producer: pphase bit s =
+// parity of the next "empty" completion of stage s to wait for.  Consumers:
+// cphase bit s = parity of the next "full" completion.
+struct Pipe {
+    uint64_t* full;   // [S] TMA completion (count 1: the producer's arrive)
+    uint64_t* empty;  // [S] stage released (count 8: one arrive per consumer warp)
+    unsigned pphase;
+    unsigned cphase;
+};
+
+// Producer: requests the weights of this CTA's first S units of a projection
+// before the grid barrier (they do not depend on the previous op).
+template <int P>
+__device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, Pipe& pp, int* err) {
+    int u_begin, n_my;
+    my_units(a.n_units, &u_begin, &n_my);
+    if (threadIdx.x == kConsumers) {
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        for (int s = 0; s < S && s < n_my; ++s) {
+            if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return false;
+            pp.pphase ^= 1u << s;
+            tma_weights<P>(a, epi, u_begin + s, smem + s * GemmSmem<P>::STAGE, pp.full + s);
+        }
+    }
+    return true;
+}
+
+// Returns false if a TMA wait timed out (error recorded).  The producer warp
+// (one elected thread) streams this CTA's units through the S stages; the 8
+// consumer warps compute and release each stage with one arrival per warp.
+template <int P>
+__device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefetched, unsigned char* smem,
+                        float* r_s, Pipe& pp, int* err) {
+    using L = GemmSmem<P>;
+    constexpr int NT = 2 * (P / 8), RC = L::RC;
+    float* red = reinterpret_cast<float*>(smem + S * L::STAGE);  // [64][RC]
+    float* ys = red + kTileRows * RC;                             // [64][16]
+    __shared__ int s_last;
+
+    const long long U = a.n_units, G = op_ctas(U);
+    const int b = blockIdx.x;
+    int u_begin, n_my;
+    my_units(U, &u_begin, &n_my);
+
+    if (threadIdx.x >= kConsumers) {  // producer warp
+        if (threadIdx.x != kConsumers) return true;
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        for (int i = 0; i < n_my; ++i) {
+            const int s = i % S;
+            unsigned char* st = smem + s * L::STAGE;
+            if (!(prefetched && i < S)) {
+                if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return false;
+                pp.pphase ^= 1u << s;
+                tma_weights<P>(a, epi, u_begin + i, st, pp.full + s);
+            }
+            tma_inputs<P>(a, M, u_begin + i, st, pp.full + s);
+        }
+        return true;
+    }
+
+    if (threadIdx.x < M) {
+        float r = 1.f;
+        if (a.ss_in) {
+            float sum = 0.f;
+            for (int t = 0; t < a.ss_in_tiles; ++t) sum += __ldcg(a.ss_in + threadIdx.x * a.ss_in_tiles + t);
+            r = rsqrtf(sum * a.inv_dim + a.eps);
+        }
+        r_s[threadIdx.x] = r;
+    }
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int rg = warp & 3, kh = warp >> 2;
+    const int g = lane >> 2, tig = lane & 3;
+    const int r0 = rg * 16 + g;
+    // two accumulator sets (k32 blocks kh, kh+4 | kh+2, kh+6) halve the MMA chain
+    float acc[NT][4], acc2[NT][4];
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+        acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = acc2[nt][0] = acc2[nt][1] = acc2[nt][2] =
+            acc2[nt][3] = 0.f;
+
+    for (int i = 0; i < n_my; ++i) {
+        const int u = u_begin + i;
+        const int tile = u / a.n_chunks, chunk = u - tile * a.n_chunks;
+        const int kc_eff = min(KC, a.K - chunk * KC);
+        const int s = i % S;
+        const unsigned char* w_s = smem + s * L::STAGE;
+        const unsigned char* x_s = w_s + L::WB;
+        if (!mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err)) return false;
+        pp.cphase ^= 1u << s;
+
+        // k32 block kb: k-box kb/2; thread tig reads 16-byte chunk 2*tig + (kb & 1)
+        // of its rows (A: weight rows r0, r0 + 8; B: input rows nt*8 + g); both
+        // operands use the same chunk -> logical-k mapping.  Columns past K are
+        // zero-filled by TMA in both operands.
+        const int nb = (kc_eff + 31) >> 5;
+        auto block = [&](int kb, float (&ac)[NT][4]) {
+            const int ch = ((2 * tig + (kb & 1)) ^ g) * 16;
+            const unsigned char* wk = w_s + (kb >> 1) * 8192;
+            const unsigned char* xk = x_s + (kb >> 1) * L::XKB;
+            const uint4 wa = *reinterpret_cast<const uint4*>(wk + r0 * 128 + ch);
+            const uint4 wb = *reinterpret_cast<const uint4*>(wk + (r0 + 8) * 128 + ch);
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+                const uint4 xv = *reinterpret_cast<const uint4*>(xk + (nt * 8 + g) * 128 + ch);
+                mma_bf16_16816(ac[nt], wa.x, wb.x, wa.y, wb.y, xv.x, xv.y);
+                mma_bf16_16816(ac[nt], wa.z, wb.z, wa.w, wb.w, xv.z, xv.w);
+            }
+        };
+        for (int kb = kh; kb < nb; kb += 4) {
+            block(kb, acc);
+            if (kb + 2 < nb) block(kb + 2, acc2);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(pp.empty + s);  // this warp is done with the stage
+
+        if (!(i == n_my - 1 || chunk == a.n_chunks - 1)) continue;
+
+        // this CTA's segment of the tile is complete: accumulator sets, then
+        // k-interleaves, then hi + lo
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                acc[nt][e] = acc[nt][e] + acc2[nt][e];
+                acc2[nt][e] = 0.f;
+            }
+        if (kh == 1) {
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+                const int c = nt * 8 + 2 * tig;
+                red[r0 * RC + c] = acc[nt][0];
+                red[r0 * RC + c + 1] = acc[nt][1];
+                red[(r0 + 8) * RC + c] = acc[nt][2];
+                red[(r0 + 8) * RC + c + 1] = acc[nt][3];
+            }
+        }
+        consumer_sync();
+        if (kh == 0) {
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+                const int c = nt * 8 + 2 * tig;
+                red[r0 * RC + c] = acc[nt][0] + red[r0 * RC + c];
+                red[r0 * RC + c + 1] = acc[nt][1] + red[r0 * RC + c + 1];
+                red[(r0 + 8) * RC + c] = acc[nt][2] + red[(r0 + 8) * RC + c];
+                red[(r0 + 8) * RC + c + 1] = acc[nt][3] + red[(r0 + 8) * RC + c + 1];
+            }
+        }
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
+        consumer_sync();
+        for (int idx = threadIdx.x; idx < kTileRows * M; idx += kGemmThreads) {
+            const int m = idx / kTileRows, r = idx - m * kTileRows;
+            ys[r * 16 + m] = red[r * RC + m] + red[r * RC + P + m];
+        }
+        consumer_sync();
+
+        // segments of other CTAs: the last one to arrive sums all in order
+        const long long u_first = (long long)tile * a.n_chunks;
+        const int seg0 = unit_owner(u_first, U, G);
+        const int nseg = unit_owner(u_first + a.n_chunks - 1, U, G) - seg0 + 1;
+        if (nseg > 1) {
+            float* slots = a.partial + (size_t)tile * a.n_chunks * kMaxRows * kTileRows;
+            float* mine = slots + (size_t)(b - seg0) * kMaxRows * kTileRows;
+            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+                const int m = idx / kTileRows, r = idx - m * kTileRows;
+                mine[m * kTileRows + r] = ys[r * 16 + m];
+            }
+            __threadfence();
+            consumer_sync();
+            if (threadIdx.x == 0) {
+                const unsigned prev = atomicAdd(&a.counters[tile], 1u);
+                s_last = prev == (unsigned)(nseg - 1);
+            }
+            consumer_sync();
+            if (!s_last) continue;
+            __threadfence();
+            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+                const int m = idx / kTileRows, r = idx - m * kTileRows;
+                const float* p = slots + m * kTileRows + r;
+                float sum = __ldcg(p);
+                for (int sg = 1; sg < nseg; ++sg) sum += __ldcg(p + (size_t)sg * kMaxRows * kTileRows);
+                ys[r * 16 + m] = sum;
+            }
+            if (threadIdx.x == 0) a.counters[tile] = 0u;
+            consumer_sync();
+        }
+
+        // epilogue of the finished tile (row m scaled by its RMSNorm factor)
+        if (epi == EPI_LOGITS) {
+            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+                const int m = idx / kTileRows, r = idx - m * kTileRows;
+                const int n = tile * kTileRows + r;
+                if (n < a.N) a.out_f32[(size_t)m * a.ldo + n] = ys[r * 16 + m] * r_s[m];
+            }
+        } else if (epi == EPI_RESID) {
+            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+                const int m = idx / kTileRows, r = idx - m * kTileRows;
+                const int n = tile * kTileRows + r;
+                float hv = 0.f;
+                if (n < a.N) {
+                    float* o = a.out_f32 + (size_t)m * a.ldo + n;
+                    hv = __ldcg(o) + ys[r * 16 + m];  // L2: other CTAs wrote h in earlier ops
+                    *o = hv;
+                    if (a.g_next) {
+                        const float z = hv * __bfloat162float(a.g_next[n]);
+                        const bf16 zh = __float2bfloat16_rn(z);
+                        a.xo_hi[(size_t)m * a.N + n] = zh;
+                        a.xo_lo[(size_t)m * a.N + n] = __float2bfloat16_rn(z - __bfloat162float(zh));
+                    }
+                }
+                ys[r * 16 + m] = hv * hv;
+            }
+            if (a.g_next) {
+                consumer_sync();
+                for (int m = warp; m < M; m += kGemmThreads / 32) {
+                    const float sq = warp_sum(ys[lane * 16 + m] + ys[(lane + 32) * 16 + m]);
+                    if (lane == 0) a.ss_out[m * a.n_tiles + tile] = sq;
+                }
+            }
+        } else if (epi == EPI_SWIGLU) {
+            for (int idx = threadIdx.x; idx < M * 32; idx += kGemmThreads) {
+                const int m = idx >> 5, r = idx & 31;
+                const int i2 = tile * 32 + r;
+                if (i2 >= a.ffn) continue;
+                const float gt = ys[r * 16 + m] * r_s[m], up = ys[(r + 32) * 16 + m] * r_s[m];
+                const float act = gt / (1.f + expf(-gt)) * up;
+                const bf16 ah = __float2bfloat16_rn(act);
+                a.xo_hi[(size_t)m * a.ffn + i2] = ah;
+                a.xo_lo[(size_t)m * a.ffn + i2] = __float2bfloat16_rn(act - __bfloat162float(ah));
+            }
+        } else {  // EPI_QKV
+            const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
+            const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
+            if (tile < q_tiles + k_tiles) {
+                const bool is_q = tile < q_tiles;
+                const int tt = is_q ? tile : tile - q_tiles;
+                const int head = tt / per_head, j0 = (tt % per_head) * 32;
+                for (int idx = threadIdx.x; idx < M * 32; idx += kGemmThreads) {
+                    const int m = idx >> 5, r = idx & 31;
+                    const int ii = j0 + r, pos = pos0 + m;
+                    const float x1 = ys[r * 16 + m] * r_s[m], x2 = ys[(r + 32) * 16 + m] * r_s[m];
+                    const float2 cs = a.rope[(size_t)pos * half + ii];
+                    const float y1 = x1 * cs.x - x2 * cs.y;
+                    const float y2 = x2 * cs.x + x1 * cs.y;
+                    if (is_q) {
+                        float* q = a.q_out + (size_t)m * a.n_heads * hd + head * hd;
+                        q[ii] = y1;
+                        q[ii + half] = y2;
+                    } else {
+                        f16* k = a.k_cache + ((size_t)head * a.max_seq + pos) * hd;
+                        k[ii] = __float2half_rn(y1);
+                        k[ii + half] = __float2half_rn(y2);
+                    }
+                }
+            } else {
+                const int vt = tile - q_tiles - k_tiles;
+                for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+                    const int m = idx / kTileRows, r = idx - m * kTileRows;
+                    const int f = vt * kTileRows + r;
+                    const int head = f / hd, e = f - head * hd;
+                    a.v_cache[((size_t)head * a.max_seq + pos0 + m) * hd + e] =
+                        __float2half_rn(ys[r * 16 + m] * r_s[m]);
+                }
+            }
+        }
+        consumer_sync();  // ys / red are reused by the next segment
+    }
+    consumer_sync();
+    return true;
+}
+
+// ---------------------------------------------------------------------------
+// attention op: units (KV head, 64-position chunk)
+// ---------------------------------------------------------------------------
+template <int HD>
+__device__ void attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem) {
+    constexpr int KP = HD * 2 + 16;  // bytes per cached row in smem (conflict-free)
+    constexpr int EPL = HD / 32;     // output dims per lane
+    constexpr int CPR = HD * 2 / 16;
+    const int G = a.n_heads / a.n_kv_heads, NV = G * M;
+    const int n_ch = (pos0 + M + kAttnChunk - 1) / kAttnChunk;  // chunks holding any visible position
+    const long long U = (long long)a.n_kv_heads * n_ch, GR = gridDim.x;
+    const int u_begin = (int)((long long)blockIdx.x * U / GR);
+    const int u_end = (int)((long long)(blockIdx.x + 1) * U / GR);
+    unsigned char* ks = smem;
+    unsigned char* vs = ks + kAttnChunk * KP;
+    float* qs = reinterpret_cast<float*>(vs + kAttnChunk * KP);  // [NV][HD]
+    float* sc = qs + NV * HD;                                     // [8][64]
+    __shared__ int s_last;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    for (int u = u_begin; u < u_end; ++u) {
+        const int kvh = u / n_ch, c = u - kvh * n_ch;
+        const int t0 = c * kAttnChunk;
+        const int t_end = min(t0 + kAttnChunk, pos0 + M);
+        float* part = a.part + ((size_t)kvh * a.n_chunks) * NV * (HD + 2);
+        const int nt = t_end - t0;
+        const f16* kb = a.k_cache + ((size_t)kvh * a.max_seq + t0) * HD;
+        const f16* vb = a.v_cache + ((size_t)kvh * a.max_seq + t0) * HD;
+        const bool wk = threadIdx.x < kAttnThreads;  // the producer warp only joins the barriers
+        for (int i = wk ? threadIdx.x : nt * CPR; i < nt * CPR; i += kAttnThreads) {
+            const int t = i / CPR, cc = i - t * CPR;
+            cp_async16(ks + t * KP + cc * 16, kb + (size_t)t * HD + cc * 8, 16);
+            cp_async16(vs + t * KP + cc * 16, vb + (size_t)t * HD + cc * 8, 16);
+        }
+        cp_async_commit();
+        for (int i = wk ? threadIdx.x : NV * HD; i < NV * HD; i += kAttnThreads) {
+            const int v = i / HD, e = i - v * HD;
+            const int m = v / G, gi = v - m * G;
+            qs[i] = __ldcg(a.q + (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e);
+        }
+        cp_async_wait<0>();
+        __syncthreads();
+
+        for (int v = wk ? warp : NV; v < NV; v += kAttnThreads / 32) {
+            const int m = v / G;
+            const int n_t = min(t_end, pos0 + m + 1) - t0;  // positions this row sees here
+            float* out = part + ((size_t)c * NV + v) * (HD + 2);
+            if (n_t <= 0) {
+                for (int e = lane; e < HD; e += 32) out[e] = 0.f;
+                if (lane == 0) { out[HD] = -INFINITY; out[HD + 1] = 0.f; }
+                continue;
+            }
+            const float* q = qs + v * HD;
+            float s[2];
+#pragma unroll
+            for (int i = 0; i < 2; ++i) {
+                const int t = lane + 32 * i;
+                float dot = -INFINITY;
+                if (t < n_t) {
+                    dot = 0.f;
+                    const unsigned char* kr = ks + t * KP;
+#pragma unroll
+                    for (int e8 = 0; e8 < HD / 8; ++e8) {
+                        const uint4 kv = *reinterpret_cast<const uint4*>(kr + e8 * 16);
+                        const float* qq = q + e8 * 8;
+                        const float2 k0 = f16x2(kv.x), k1 = f16x2(kv.y), k2 = f16x2(kv.z), k3 = f16x2(kv.w);
+                        dot += qq[0] * k0.x + qq[1] * k0.y;
+                        dot += qq[2] * k1.x + qq[3] * k1.y;
+                        dot += qq[4] * k2.x + qq[5] * k2.y;
+                        dot += qq[6] * k3.x + qq[7] * k3.y;
+                    }
+                    dot *= a.scale;
+                }
+                s[i] = dot;
+            }
+            const float mx = warp_max(fmaxf(s[0], s[1]));
+            const float p0 = lane < n_t ? expf(s[0] - mx) : 0.f;
+            const float p1 = lane + 32 < n_t ? expf(s[1] - mx) : 0.f;
+            const float l = warp_sum(p0 + p1);
+            float* sw = sc + warp * kAttnChunk;
+            sw[lane] = p0;
+            sw[lane + 32] = p1;
+            __syncwarp();
+            float o[EPL];
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) o[e] = 0.f;
+            for (int t = 0; t < n_t; ++t) {
+                const float w = sw[t];
+                const unsigned char* vr = vs + t * KP + lane * EPL * 2;
+                if constexpr (EPL == 4) {
+                    const uint2 vv = *reinterpret_cast<const uint2*>(vr);
+                    const float2 v0 = f16x2(vv.x), v1 = f16x2(vv.y);
+                    o[0] += w * v0.x;
+                    o[1] += w * v0.y;
+                    o[2] += w * v1.x;
+                    o[3] += w * v1.y;
+                } else {
+                    const float2 v0 = f16x2(*reinterpret_cast<const uint32_t*>(vr));
+                    o[0] += w * v0.x;
+                    o[1] += w * v0.y;
+                }
+            }
+            __syncwarp();
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) out[lane * EPL + e] = o[e];
+            if (lane == 0) { out[HD] = mx; out[HD + 1] = l; }
+        }
+
+        __threadfence();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const unsigned prev = atomicAdd(&a.counters[kvh], 1u);
+            s_last = prev == (unsigned)(n_ch - 1);
+        }
+        __syncthreads();
+        if (s_last) {
+            __threadfence();
+            // combine: row m uses chunks 0 .. (pos0 + m) / 64, in chunk order
+            for (int v = wk ? warp : NV; v < NV; v += kAttnThreads / 32) {
+                const int m = v / G, gi = v - m * G;
+                const int nch = (pos0 + m) / kAttnChunk + 1;
+                float mx = -INFINITY;
+                for (int cc = 0; cc < nch; ++cc)
+                    mx = fmaxf(mx, __ldcg(part + ((size_t)cc * NV + v) * (HD + 2) + HD));
+                float L = 0.f;
+                float o[EPL];
+#pragma unroll
+                for (int e = 0; e < EPL; ++e) o[e] = 0.f;
+                for (int cc = 0; cc < nch; ++cc) {
+                    const float* pp = part + ((size_t)cc * NV + v) * (HD + 2);
+                    const float mc = __ldcg(pp + HD);
+                    if (mc == -INFINITY) continue;
+                    const float f = expf(mc - mx);
+                    L += f * __ldcg(pp + HD + 1);
+#pragma unroll
+                    for (int e = 0; e < EPL; ++e) o[e] += f * __ldcg(pp + lane * EPL + e);
+                }
+                const float inv = 1.f / L;
+                const size_t at = (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + lane * EPL;
+#pragma unroll
+                for (int e = 0; e < EPL; ++e) {
+                    const float val = o[e] * inv;
+                    const bf16 vh = __float2bfloat16_rn(val);
+                    a.out_hi[at + e] = vh;
+                    a.out_lo[at + e] = __float2bfloat16_rn(val - __bfloat162float(vh));
+                }
+            }
+            if (threadIdx.x == 0) a.counters[kvh] = 0u;
+        }
+        __syncthreads();  // smem reused by the next unit
+    }
+}
+
+// ---------------------------------------------------------------------------
+// embedding op: h = E[token], planes of h * g (first RMSNorm), sums of h^2
+// ---------------------------------------------------------------------------
+__device__ void embed_op(const FwdParams& p, int pos0) {
+    if (threadIdx.x >= kConsumers) return;
+    const int d = p.d, n_tiles = d / 64;
+    const int lane = threadIdx.x & 31;
+    const int gw = blockIdx.x * (kGemmThreads / 32) + (threadIdx.x >> 5);
+    const int nw = gridDim.x * (kGemmThreads / 32);
+    if (blockIdx.x == 0 && threadIdx.x == 0) p.st->pos0 = pos0;
+    for (int u = gw; u < p.M * n_tiles; u += nw) {
+        const int m = u / n_tiles, t = u - m * n_tiles;
+        int tok;
+        if (p.src == SRC_TOKENS) tok = p.toks[m];
+        else if (p.src == SRC_DRAFT) tok = p.st->j == 0 ? p.st->x_last : p.st->drafts[p.st->j - 1];
+        else tok = m == 0 ? p.st->x_last : p.st->drafts[m - 1];
+        const bf16* row = p.embed + (size_t)tok * d;
+        float sq = 0.f;
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+            const int i = t * 64 + j * 32 + lane;
+            const float v = __bfloat162float(row[i]);
+            p.h[(size_t)m * d + i] = v;
+            const float z = v * __bfloat162float(p.g0[i]);
+            const bf16 zh = __float2bfloat16_rn(z);
+            p.xn_hi[(size_t)m * d + i] = zh;
+            p.xn_lo[(size_t)m * d + i] = __float2bfloat16_rn(z - __bfloat162float(zh));
+            sq += v * v;
+        }
+        sq = warp_sum(sq);
+        if (lane == 0) p.ss[m * n_tiles + t] = sq;
+    }
+}
+
+// Block-cooperative copy of an op descriptor into shared memory.
+__device__ __forceinline__ void copy_op(const FwdOp* src, FwdOp* dst) {
+    static_assert(sizeof(FwdOp) % 4 == 0, "FwdOp is copied in 4-byte words");
+    const unsigned* s = reinterpret_cast<const unsigned*>(src);
+    unsigned* d = reinterpret_cast<unsigned*>(dst);
+    for (int i = threadIdx.x; i < (int)(sizeof(FwdOp) / 4); i += blockDim.x) d[i] = s[i];
+    __syncthreads();
+}
+
+// After a timed-out wait: give copies still in flight a bounded time to land
+// before the CTA exits (the error is already recorded).
+__device__ void drain_before_exit() {
+    if (threadIdx.x == 0) {
+        const unsigned long long t0 = globaltimer();
+        while (globaltimer() - t0 < 2000000ull) __nanosleep(1000);
+    }
+    __syncthreads();
+}
+
+template <int NPH, int HD>
+__global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams p) {
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    __shared__ float r_s[kMaxRows];
+    __shared__ int s_pos0, s_fail;
+    __shared__ __align__(8) uint64_t full[S];   // TMA completion per stage
+    __shared__ __align__(8) uint64_t empty[S];  // stage released by the 8 consumer warps
+    __shared__ FwdOp s_op[2];                   // current and next op's arguments
+    constexpr int P = 8 * NPH;
+    // 128-byte TMA swizzle needs 1 KB aligned boxes
+    unsigned char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    if (threadIdx.x == 0) {
+        int pos0;
+        if (p.src == SRC_TOKENS) pos0 = p.pos0_arg;
+        else if (p.src == SRC_DRAFT) pos0 = p.st->len + p.st->j;
+        else pos0 = p.st->len;
+        s_pos0 = pos0;
+        s_fail = 0;
+        for (int st = 0; st < S; ++st) {
+            mbar_init(full + st, 1);
+            mbar_init(empty + st, kConsumers / 32);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        if (p.trace && blockIdx.x == 0) p.trace[0] = globaltimer();
+    }
+    __syncthreads();
+    // every stage starts empty: each consumer warp releases it once
+    if (threadIdx.x < kConsumers && (threadIdx.x & 31) == 0)
+        for (int st = 0; st < S; ++st) mbar_arrive(empty + st);
+    const int pos0 = s_pos0;
+    unsigned target = 0;
+    Pipe pp{full, empty, 0u, 0u};
+    bool prefetched = false;
+    copy_op(p.ops, s_op);
+    for (int o = 0; o < p.n_ops; ++o) {
+        const FwdOp& op = s_op[o & 1];
+        const int type = op.type;
+        bool ok = true;
+        if (type == OP_EMBED) embed_op(p, pos0);
+        else if (type == OP_ATTN) attn_op<HD>(op.at, p.M, pos0, smem);
+        else ok = gemm_op<P>(op.g, epi_of(type), p.M, pos0, prefetched, smem, r_s, pp, p.err);
+        prefetched = false;
+        if (o + 1 < p.n_ops) {
+            copy_op(p.ops + o + 1, s_op + ((o + 1) & 1));  // (all threads, includes a barrier)
+            const FwdOp& nx = s_op[(o + 1) & 1];
+            if (ok && is_gemm(nx.type)) {
+                ok = gemm_prefetch<P>(nx.g, epi_of(nx.type), smem, pp, p.err);
+                prefetched = true;
+            }
+        }
+        if (!ok) s_fail = 1;
+        __syncthreads();
+        if (s_fail) {
+            drain_before_exit();
+            return;
+        }
+        if (o + 1 < p.n_ops) {
+            target += gridDim.x;
+            if (!grid_barrier(p.bar, target, p.err)) {
+                drain_before_exit();
+                return;
+            }
+        }
+        if (p.trace && blockIdx.x == 0 && threadIdx.x == 0) p.trace[o + 1] = globaltimer();
+    }
+}
+
+template <int NPH, int HD>
+int launch_fwd(const FwdParams& p, int grid, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid, 1, 1);
+    cfg.blockDim = dim3(kFwdThreads, 1, 1);
+    cfg.dynamicSmemBytes = GemmSmem<8 * NPH>::BYTES;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return (int)cudaLaunchKernelEx(&cfg, forward_kernel<NPH, HD>, p);
+}
+
+template <int NPH, int HD>
+int configure_fwd() {
+    return (int)cudaFuncSetAttribute(forward_kernel<NPH, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)GemmSmem<8 * NPH>::BYTES);
+}
+
+}  // namespace
+
+size_t forward_smem_bytes(int M) { return M <= 8 ? GemmSmem<8>::BYTES : GemmSmem<16>::BYTES; }
+
+size_t attention_smem_bytes(int head_dim, int group, int M) {
+    return 2 * kAttnChunk * (head_dim * 2 + 16) + (size_t)group * M * head_dim * 4 + 8 * kAttnChunk * 4;
+}
+
+int forward_configure() {
+    int e = 0;
+    e = e ? e : configure_fwd<1, 64>();
+    e = e ? e : configure_fwd<2, 64>();
+    e = e ? e : configure_fwd<1, 128>();
+    e = e ? e : configure_fwd<2, 128>();
+    return e;
+}
+
+int launch_forward(const FwdParams& p, int head_dim, int grid, cudaStream_t s) {
+    const bool two = p.M > 8;
+    if (head_dim == 128) return two ? launch_fwd<2, 128>(p, grid, s) : launch_fwd<1, 128>(p, grid, s);
+    if (head_dim == 64) return two ? launch_fwd<2, 64>(p, grid, s) : launch_fwd<1, 64>(p, grid, s);
+    return (int)cudaErrorInvalidValue;
+}
+
+}  // namespace ssd

@@ -37,48 +37,6 @@
 namespace ssd {
 namespace {
 
-__device__ __forceinline__ const bf16* row_src(const GemmArgs& a, int epi, int tile, int r) {
-    const int K = a.K;
-    if (epi == EPI_LOGITS || epi == EPI_RESID) {
-        int n = tile * kTileRows + r;
-        return n < a.N ? a.w0 + (size_t)n * K : nullptr;
-    }
-    if (epi == EPI_SWIGLU) {
-        int i = tile * 32 + (r & 31);
-        if (i >= a.ffn) return nullptr;
-        return (r < 32 ? a.w0 : a.w1) + (size_t)i * K;
-    }
-    // EPI_QKV: q and k tiles hold 32 RoPE pairs (i, i + hd/2) of one head
-    const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
-    const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
-    if (tile < q_tiles + k_tiles) {
-        bool is_q = tile < q_tiles;
-        int tt = is_q ? tile : tile - q_tiles;
-        int head = tt / per_head, j0 = (tt % per_head) * 32;
-        int f = head * hd + (r >> 5) * half + j0 + (r & 31);
-        return (is_q ? a.w0 : a.w1) + (size_t)f * K;
-    }
-    int f = (tile - q_tiles - k_tiles) * kTileRows + r;
-    return a.w2 + (size_t)f * K;
-}
-
-// Splits 8 fp32 activations into bf16 hi = rn(x) and lo = rn(x - hi), so that
-// W * hi + W * lo carries ~16 mantissa bits of x through the bf16 MMA.
-__device__ __forceinline__ void split8(const float4& f0, const float4& f1, uint4& hi, uint4& lo) {
-    const float f[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
-    uint32_t h[4], l[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        __nv_bfloat162 hv = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
-        float2 hf = __bfloat1622float2(hv);
-        __nv_bfloat162 lv = __floats2bfloat162_rn(f[2 * i] - hf.x, f[2 * i + 1] - hf.y);
-        h[i] = *reinterpret_cast<uint32_t*>(&hv);
-        l[i] = *reinterpret_cast<uint32_t*>(&lv);
-    }
-    hi = make_uint4(h[0], h[1], h[2], h[3]);
-    lo = make_uint4(l[0], l[1], l[2], l[3]);
-}
-
 // NPH = n8 tiles per activation half (1: M <= 8, 2: M <= 16).  The MMA's N
 // side holds P = 8*NPH rows of x_hi followed by P rows of x_lo.
 template <int NPH, int EPI>

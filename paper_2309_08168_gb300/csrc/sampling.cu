@@ -1,5 +1,5 @@
-// sampling.cu - per-row kernels around the projections: embedding gather,
-// RMSNorm, and the token choice / acceptance of self-speculative decoding:
+// sampling.cu - the token choice and acceptance kernels that follow a
+// forward in self-speculative decoding:
 //   greedy draft      x_{j+1} = argmax p(x | z*, ...)              (Algorithm 2)
 //   greedy accept     longest prefix d_j == argmax p_{j-1}; the first
 //                     mismatch is corrected, or a bonus token added (Alg. 2)
@@ -262,51 +262,6 @@ __device__ int sample_row(const float* s, int V, float u, float* red, int* redi)
 // ---------------------------------------------------------------------------
 // kernels
 // ---------------------------------------------------------------------------
-__global__ void embed_kernel(const bf16* __restrict__ E, int d, int M, int src,
-                             const int* __restrict__ toks, int pos0_arg, DecodeState* st,
-                             float* __restrict__ h) {
-    pdl_launch_dependents();
-    pdl_wait();
-    const int m = blockIdx.x;
-    int tok, pos0;
-    if (src == SRC_TOKENS) { tok = toks[m]; pos0 = pos0_arg; }
-    else if (src == SRC_DRAFT) {
-        tok = st->j == 0 ? st->x_last : st->drafts[st->j - 1];
-        pos0 = st->len + st->j;
-    } else {
-        tok = m == 0 ? st->x_last : st->drafts[m - 1];
-        pos0 = st->len;
-    }
-    __syncthreads();
-    if (m == 0 && threadIdx.x == 0) st->pos0 = pos0;
-    const bf16* row = E + (size_t)tok * d;
-    for (int i = threadIdx.x; i < d; i += blockDim.x) h[(size_t)m * d + i] = __bfloat162float(row[i]);
-}
-
-__global__ void rmsnorm_kernel(const float* __restrict__ h, const bf16* __restrict__ g, int d,
-                               float eps, float* __restrict__ out) {
-    pdl_launch_dependents();
-    pdl_wait();
-    __shared__ float red[33];
-    const int m = blockIdx.x;
-    const float* x = h + (size_t)m * d;
-    float ss = 0.f;
-    for (int i = threadIdx.x; i < d; i += blockDim.x) ss += x[i] * x[i];
-    ss = warp_sum(ss);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) red[warp] = ss;
-    __syncthreads();
-    if (warp == 0) {
-        float r = lane < (int)(blockDim.x >> 5) ? red[lane] : 0.f;
-        r = warp_sum(r);
-        if (lane == 0) red[32] = rsqrtf(r / (float)d + eps);
-    }
-    __syncthreads();
-    const float r = red[32];
-    for (int i = threadIdx.x; i < d; i += blockDim.x)
-        out[(size_t)m * d + i] = x[i] * r * __bfloat162float(g[i]);
-}
-
 // greedy drafting: d_{j+1} = argmax of the draft logits
 __global__ void __launch_bounds__(kRowThreads) greedy_draft_kernel(const float* __restrict__ logits,
                                                                    int V, DecodeState* st) {
@@ -501,9 +456,7 @@ int launch_pdl(Kern k, dim3 grid, dim3 block, size_t smem, cudaStream_t s, Args.
 int sampling_configure() {
     // load every kernel of this file now, outside any stream capture
     cudaFuncAttributes fa;
-    cudaError_t e0 = cudaFuncGetAttributes(&fa, embed_kernel);
-    if (e0 == cudaSuccess) e0 = cudaFuncGetAttributes(&fa, rmsnorm_kernel);
-    if (e0 == cudaSuccess) e0 = cudaFuncGetAttributes(&fa, greedy_draft_kernel);
+    cudaError_t e0 = cudaFuncGetAttributes(&fa, greedy_draft_kernel);
     if (e0 == cudaSuccess) e0 = cudaFuncGetAttributes(&fa, greedy_accept_kernel);
     if (e0 != cudaSuccess) return (int)e0;
     const int big = 160 * 1024;
@@ -513,16 +466,6 @@ int sampling_configure() {
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(spec_accept_batch_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, big);
     return (int)e;
-}
-
-int launch_embed(const bf16* embed, int d, int M, int src, const int* tokens_dev, int pos0,
-                 DecodeState* st, float* h, cudaStream_t s) {
-    return launch_pdl(embed_kernel, dim3(M), dim3(256), 0, s, embed, d, M, src, tokens_dev, pos0, st, h);
-}
-
-int launch_rmsnorm(const float* h, const bf16* g, int d, int M, float eps, float* out,
-                   cudaStream_t s) {
-    return launch_pdl(rmsnorm_kernel, dim3(M), dim3(512), 0, s, h, g, d, eps, out);
 }
 
 int launch_greedy_draft(const float* logits, int V, DecodeState* st, cudaStream_t s) {

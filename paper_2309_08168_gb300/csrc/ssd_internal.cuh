@@ -17,6 +17,8 @@ constexpr int kTileRows = 64;     // output rows per GEMM CTA
 constexpr int kGemmThreads = 256; // 8 warps: 4 row groups x 2 k-interleaves
 constexpr int kAttnChunk = 64;    // KV positions per attention CTA (absolute chunks)
 constexpr int kAttnThreads = 256;
+constexpr int kStreamKC = 256;    // k per streaming-GEMM work unit (64 rows x 256 = 32 KB of weights)
+constexpr int kStreamStages = 4;  // cp.async ring depth of the streaming GEMM
 
 // ---------------------------------------------------------------------------
 // device state of the decode loop (one per handle, in device memory)
@@ -68,6 +70,20 @@ struct GemmArgs {
     const float2* rope;  // [max_seq][hd/2] (cos, sin)
     const DecodeState* st;  // pos0
     int* err;            // device error flag (checked builds)
+    // streaming GEMM (gemm_stream.cu)
+    const bf16* x_hi;    // input planes [M][K]: bf16 hi = rn(v), lo = rn(v - hi)
+    const bf16* x_lo;
+    const float* ss_in;  // [M][ss_in_tiles] sums of squares of the pre-norm row (nullptr: no norm)
+    int ss_in_tiles;
+    float inv_dim, eps;  // RMSNorm scale of row m: rsqrt(sum(ss_in[m]) * inv_dim + eps)
+    const bf16* g_next;  // EPI_RESID: gains of the next RMSNorm (nullptr: no next input)
+    bf16* xo_hi;         // EPI_RESID: planes of h * g_next [M][N]; EPI_SWIGLU: act planes [M][ffn]
+    bf16* xo_lo;
+    float* ss_out;       // EPI_RESID: [M][n_tiles] per-tile sums of h^2
+    int n_chunks;        // ceil(K / kStreamKC)
+    int n_units;         // n_tiles * n_chunks
+    const void* tm_w[3];     // TMA tensor maps (global memory) of w0, w1, w2: box 64 k x 32 rows
+    const void* tm_x[3][2];  // TMA maps of the input planes [box rows 1 | 8 | 16][hi | lo]
 };
 
 // ---------------------------------------------------------------------------
@@ -78,7 +94,8 @@ struct AttnArgs {
     const float* q;      // [M][H*hd]
     const f16* k_cache;  // [Hkv][max_seq][hd] fp16
     const f16* v_cache;
-    float* out;          // [M][H*hd]
+    bf16* out_hi;        // [M][H*hd] output planes: hi = rn(o), lo = rn(o - hi)
+    bf16* out_lo;
     float* part;         // [Hkv][n_chunks][G*M][hd + 2]
     unsigned* counters;  // [Hkv]
     int M, n_heads, n_kv_heads, head_dim, max_seq, n_chunks;
@@ -87,21 +104,54 @@ struct AttnArgs {
     int* err;            // device error flag (checked builds)
 };
 
+// ---------------------------------------------------------------------------
+// forward kernel (forward_kernel.cu): one persistent cooperative launch per
+// decoder forward, walking a device-resident op list
+// ---------------------------------------------------------------------------
+enum OpType { OP_EMBED = 0, OP_QKV = 1, OP_ATTN = 2, OP_RESID = 3, OP_SWIGLU = 4, OP_LOGITS = 5 };
+constexpr int kDevErrTimeout = 1;  // DecodeState::err: a grid barrier or a TMA wait gave up
+
+struct FwdOp {
+    int type;
+    GemmArgs g;   // projection ops
+    AttnArgs at;  // attention op
+};
+
+struct FwdParams {
+    const FwdOp* ops;
+    int n_ops;
+    int M;                // rows of this forward (1..16)
+    int src;              // EmbedSrc: where the tokens and the first position come from
+    const int* toks;      // SRC_TOKENS: device token ids
+    int pos0_arg;         // SRC_TOKENS: first position
+    DecodeState* st;
+    const bf16* embed;
+    int d;
+    const bf16* g0;       // gains of the first RMSNorm that runs
+    float* h;             // residual stream [16][d]
+    bf16* xn_hi;          // planes of h * g [16][d]
+    bf16* xn_lo;
+    float* ss;            // per-64-column sums of h^2 [16][d/64]
+    unsigned* bar;        // grid-barrier counter, zero at launch
+    int* err;             // device error code
+    unsigned long long* trace;  // nullptr, or [n_ops + 1] globaltimer stamps (start, end of op o)
+};
+
+int forward_configure();
+size_t forward_smem_bytes(int M);
+size_t attention_smem_bytes(int head_dim, int group, int M);
+int launch_forward(const FwdParams& p, int head_dim, int grid, cudaStream_t s);
+
 // sets the thread's ssd_last_error() message and returns code
 int set_last_error(int code, const char* msg);
 
 // launchers (return cudaError_t)
 int gemm_configure();
-int attention_configure();
 int launch_gemm(int epi, const GemmArgs& a, cudaStream_t s);
-int launch_attention(const AttnArgs& a, cudaStream_t s);
 size_t gemm_smem_bytes(int kc, int M);
 constexpr int gemm_half_rows(int M) { return M <= 8 ? 8 : 16; }  // padded rows of x_hi (and of x_lo)
 
-int launch_embed(const bf16* embed, int d, int M, int src, const int* tokens_dev, int pos0,
-                 DecodeState* st, float* h, cudaStream_t s);
-int launch_rmsnorm(const float* h, const bf16* g, int d, int M, float eps, float* out,
-                   cudaStream_t s);
+
 
 // src for launch_embed
 enum EmbedSrc { SRC_TOKENS = 0, SRC_DRAFT = 1, SRC_VERIFY = 2 };
@@ -176,6 +226,51 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint3
         "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
         : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// ---------------------------------------------------------------------------
+// GEMM helpers shared by both GEMM kernels
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ const bf16* row_src(const GemmArgs& a, int epi, int tile, int r) {
+    const int K = a.K;
+    if (epi == EPI_LOGITS || epi == EPI_RESID) {
+        int n = tile * kTileRows + r;
+        return n < a.N ? a.w0 + (size_t)n * K : nullptr;
+    }
+    if (epi == EPI_SWIGLU) {
+        int i = tile * 32 + (r & 31);
+        if (i >= a.ffn) return nullptr;
+        return (r < 32 ? a.w0 : a.w1) + (size_t)i * K;
+    }
+    // EPI_QKV: q and k tiles hold 32 RoPE pairs (i, i + hd/2) of one head
+    const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
+    const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
+    if (tile < q_tiles + k_tiles) {
+        bool is_q = tile < q_tiles;
+        int tt = is_q ? tile : tile - q_tiles;
+        int head = tt / per_head, j0 = (tt % per_head) * 32;
+        int f = head * hd + (r >> 5) * half + j0 + (r & 31);
+        return (is_q ? a.w0 : a.w1) + (size_t)f * K;
+    }
+    int f = (tile - q_tiles - k_tiles) * kTileRows + r;
+    return a.w2 + (size_t)f * K;
+}
+
+// Splits 8 fp32 activations into bf16 hi = rn(x) and lo = rn(x - hi), so that
+// W * hi + W * lo carries ~16 mantissa bits of x through the bf16 MMA.
+__device__ __forceinline__ void split8(const float4& f0, const float4& f1, uint4& hi, uint4& lo) {
+    const float f[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        __nv_bfloat162 hv = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
+        float2 hf = __bfloat1622float2(hv);
+        __nv_bfloat162 lv = __floats2bfloat162_rn(f[2 * i] - hf.x, f[2 * i + 1] - hf.y);
+        h[i] = *reinterpret_cast<uint32_t*>(&hv);
+        l[i] = *reinterpret_cast<uint32_t*>(&lv);
+    }
+    hi = make_uint4(h[0], h[1], h[2], h[3]);
+    lo = make_uint4(l[0], l[1], l[2], l[3]);
 }
 
 }  // namespace ssd
