@@ -82,7 +82,7 @@ def _load():
     lib.ssd_debug_spec_accept.argtypes = [H, _VP, _VP, ctypes.c_int, _VP, _VP, ctypes.c_int, ctypes.c_int, _VP]
     lib.ssd_debug_time_forward.argtypes = [H, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                            _VP, _VP, _VP]
-    lib.ssd_debug_trace_forward.argtypes = [H, ctypes.c_int, ctypes.c_int, _VP, _VP, ctypes.c_int, _VP]
+    lib.ssd_debug_trace_forward.argtypes = [H, ctypes.c_int, ctypes.c_int, _VP, _VP, ctypes.c_int, _VP, _VP]
     lib.ssd_debug_trace_forward.restype = ctypes.c_int
     lib.ssd_linear_noalloc.argtypes = [_VP, _VP, _VP, ctypes.c_int, ctypes.c_int, ctypes.c_int, _VP]
     lib.ssd_linear_noalloc.restype = ctypes.c_int
@@ -186,16 +186,20 @@ def ssd_linear_noalloc(w, x, y, N: int, K: int, M: int, cuda_stream: int | None 
 OP_NAMES = ("embed", "qkv", "attention", "o/down", "gate/up", "lm_head")
 
 
-def ssd_debug_trace_forward(h: int, draft: bool, rows: int):
-    """Returns [(op name, microseconds)] for one forward of the forward kernel."""
+def ssd_debug_trace_forward(h: int, draft: bool, rows: int, units: bool = False):
+    """Returns [(op name, microseconds)] for one forward of the forward kernel
+    (and, with units=True, also the [64][4] unit stamps of CTA 0's first
+    projection, in ns)."""
     cfg = config_of(h)
     cap = 2 + 5 * cfg.n_layers
     us = np.zeros(cap, dtype=np.float32)
     ty = np.zeros(cap, dtype=np.int32)
+    ut = np.zeros((64, 4), dtype=np.uint64)
     n = ctypes.c_int()
     _check(lib.ssd_debug_trace_forward(h, int(draft), rows, us.ctypes.data, ty.ctypes.data, cap,
-                                       ctypes.addressof(n)))
-    return [(OP_NAMES[ty[i]], float(us[i])) for i in range(n.value)]
+                                       ctypes.addressof(n), ut.ctypes.data))
+    ops = [(OP_NAMES[ty[i]], float(us[i])) for i in range(n.value)]
+    return (ops, ut) if units else ops
 
 
 def ssd_destroy(h: int) -> None:
@@ -282,5 +286,5 @@ class Decoder:
     def debug_time_forward(self, draft, rows, gemm_only, reps):
         return ssd_debug_time_forward(self.h, draft, rows, gemm_only, reps)
 
-    def debug_trace_forward(self, draft, rows):
-        return ssd_debug_trace_forward(self.h, draft, rows)
+    def debug_trace_forward(self, draft, rows, units=False):
+        return ssd_debug_trace_forward(self.h, draft, rows, units)

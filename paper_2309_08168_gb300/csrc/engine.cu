@@ -103,8 +103,8 @@ struct ssd_handle {
     f16* vc = nullptr;
     size_t kv_layer = 0;  // elements per layer of one of K / V
     float* h = nullptr;
-    bf16* xn_hi = nullptr;  // planes of h * g (input of the next normed projection) [16][d]
-    bf16* xn_lo = nullptr;
+    bf16* xn_hi = nullptr;  // planes of h * g (input of the next normed projection) [2][16][d]
+    bf16* xn_lo = nullptr;  // = xn_hi + 16 * d
     float* ss = nullptr;    // per-64-column sums of h^2 [16][d/64]
     float* q = nullptr;
     bf16* at_hi = nullptr;  // attention output planes [16][H*hd]
@@ -174,31 +174,60 @@ const bf16* next_norm(const ssd_handle* h, int s, bool draft) {
 
 // ---------------------------------------------------------------------------
 // TMA descriptors.  Index layout: layer l's wq wk wv wo w_gate w_up w_down at
-// 7l + 0..6, lm_head at 7L, then the input planes: 7L + 1 + (buf * 3 + cls) * 2
-// + plane with buf 0 = normalised rows (K = d), 1 = attention output (K = H*hd),
-// 2 = SwiGLU output (K = ffn); cls = box rows 1 | 8 | 16; plane 0 hi, 1 lo.
+// 7l + 0..6, lm_head at 7L, then the input-plane maps at 7L + 1 + buf * 3 + cls
+// with buf 0 = normalised rows (K = d), 1 = attention output (K = H*hd),
+// 2 = SwiGLU output (K = ffn) and cls = rows per plane 1 | 8 | 16.
 // ---------------------------------------------------------------------------
 int tmap_weight(int l, int which) { return 7 * l + which; }
-int tmap_x(const ssd_handle* h, int buf, int cls, int plane) {
-    return 7 * h->cfg.n_layers + 1 + (buf * 3 + cls) * 2 + plane;
-}
+int tmap_x(const ssd_handle* h, int buf, int cls) { return 7 * h->cfg.n_layers + 1 + buf * 3 + cls; }
 
-// A 2D bf16 tensor [rows][K] row-major, box 64 (k) x box_rows, 128-byte swizzle,
-// out-of-range elements read as zero.  Checks the TMA rules: 16-byte aligned
-// base, row stride a multiple of 16 bytes, 128-byte inner box.
-int encode_map(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* base, int K, int rows,
-               int box_rows) {
-    if (((uintptr_t)base & 15u) || ((K * 2) % 16) || K < 64 || box_rows < 1 || box_rows > 256)
-        return fail(SSD_ERR_INVALID_ARG, "tensor not suitable for TMA (alignment / row length)");
-    cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)K * 2};
-    cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
-    cuuint32_t estr[2] = {1, 1};
-    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+// Checks the TMA rules and encodes a bf16 tensor map with 64-element (128-byte)
+// inner boxes, 128-byte swizzle, zero fill out of range: base 16-byte aligned,
+// strides multiples of 16 bytes.
+int encode_map(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* base, int rank,
+               const cuuint64_t* dims, const cuuint64_t* strides, const cuuint32_t* box) {
+    if ((uintptr_t)base & 15u) return fail(SSD_ERR_INVALID_ARG, "tensor base not 16-byte aligned for TMA");
+    for (int i = 0; i + 1 < rank; ++i)
+        if (strides[i] % 16) return fail(SSD_ERR_INVALID_ARG, "tensor stride not a multiple of 16 bytes for TMA");
+    if (dims[0] < 64 || box[0] != 64) return fail(SSD_ERR_INVALID_ARG, "tensor row shorter than one TMA box");
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base), dims, strides,
+                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return fail(SSD_ERR_CUDA, "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")");
     return SSD_OK;
+}
+
+// weight matrix [rows][K] bf16.  K % 64 == 0: viewed as {64, K/64, rows} with
+// box {64, 4, 32} (a 64-row x 256-k unit is two copies); otherwise 2D with box
+// 64 (k) x 32 rows (eight copies per unit).
+int encode_weight(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* base, int K, int rows) {
+    if (K % 64 == 0) {
+        cuuint64_t dims[3] = {64, (cuuint64_t)K / 64, (cuuint64_t)rows};
+        cuuint64_t strides[2] = {128, (cuuint64_t)K * 2};
+        cuuint32_t box[3] = {64, 4, 32};
+        return encode_map(enc, m, base, 3, dims, strides, box);
+    }
+    cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+    cuuint32_t box[2] = {64, 32};
+    return encode_map(enc, m, base, 2, dims, strides, box);
+}
+
+// input planes [2][16][K] bf16 (hi plane, lo plane).  K % 64 == 0: viewed as
+// {64, K/64, 16, 2} with box {64, 4, R, 2} (one copy per unit); otherwise 3D
+// {K, 16, 2} with box {64, R, 2} (one copy per 64-wide k-box).
+int encode_planes(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* base, int K, int R) {
+    if (K % 64 == 0) {
+        cuuint64_t dims[4] = {64, (cuuint64_t)K / 64, (cuuint64_t)kMaxRows, 2};
+        cuuint64_t strides[3] = {128, (cuuint64_t)K * 2, (cuuint64_t)K * 2 * kMaxRows};
+        cuuint32_t box[4] = {64, 4, (cuuint32_t)R, 2};
+        return encode_map(enc, m, base, 4, dims, strides, box);
+    }
+    cuuint64_t dims[3] = {(cuuint64_t)K, (cuuint64_t)kMaxRows, 2};
+    cuuint64_t strides[2] = {(cuuint64_t)K * 2, (cuuint64_t)K * 2 * kMaxRows};
+    cuuint32_t box[3] = {64, (cuuint32_t)R, 2};
+    return encode_map(enc, m, base, 3, dims, strides, box);
 }
 
 int build_tmaps(ssd_handle* h) {
@@ -216,16 +245,15 @@ int build_tmaps(ssd_handle* h) {
         const bf16* w[7] = {h->wq[l], h->wk[l], h->wv[l], h->wo[l], h->w_gate[l], h->w_up[l], h->w_down[l]};
         const int K[7] = {d, d, d, qd, d, d, c.ffn};
         const int N[7] = {qd, kvd, kvd, d, c.ffn, c.ffn, d};
-        for (int i = 0; i < 7 && !rc; ++i) rc = encode_map(enc, &maps[tmap_weight(l, i)], w[i], K[i], N[i], 32);
+        for (int i = 0; i < 7 && !rc; ++i) rc = encode_weight(enc, &maps[tmap_weight(l, i)], w[i], K[i], N[i]);
     }
-    if (!rc) rc = encode_map(enc, &maps[7 * L], h->lm_head, d, c.vocab, 32);
-    const bf16* planes[3][2] = {{h->xn_hi, h->xn_lo}, {h->at_hi, h->at_lo}, {h->ac_hi, h->ac_lo}};
+    if (!rc) rc = encode_weight(enc, &maps[7 * L], h->lm_head, d, c.vocab);
+    const bf16* planes[3] = {h->xn_hi, h->at_hi, h->ac_hi};
     const int widths[3] = {d, qd, c.ffn};
-    const int heights[3] = {1, 8, 16};
+    const int rows[3] = {1, 8, 16};
     for (int b = 0; b < 3 && !rc; ++b)
         for (int cls = 0; cls < 3 && !rc; ++cls)
-            for (int pl = 0; pl < 2 && !rc; ++pl)
-                rc = encode_map(enc, &maps[tmap_x(h, b, cls, pl)], planes[b][pl], widths[b], kMaxRows, heights[cls]);
+            rc = encode_planes(enc, &maps[tmap_x(h, b, cls)], planes[b], widths[b], rows[cls]);
     if (rc) return rc;
     CUDA_TRY(cudaMemcpy(h->tmaps, maps.data(), maps.size() * sizeof(CUtensorMap), cudaMemcpyHostToDevice),
              "tensor map upload");
@@ -233,8 +261,7 @@ int build_tmaps(ssd_handle* h) {
 }
 
 void set_x_maps(const ssd_handle* h, GemmArgs& a, int buf) {
-    for (int cls = 0; cls < 3; ++cls)
-        for (int pl = 0; pl < 2; ++pl) a.tm_x[cls][pl] = h->tmaps + tmap_x(h, buf, cls, pl);
+    for (int cls = 0; cls < 3; ++cls) a.tm_x[cls] = h->tmaps + tmap_x(h, buf, cls);
 }
 
 // One projection op: fills the fields every projection shares.
@@ -244,6 +271,7 @@ GemmArgs proj_args(ssd_handle* h, int N, int K, int n_tiles, const bf16* x_hi, c
     a.K = K;
     a.n_tiles = n_tiles;
     a.n_chunks = (K + kStreamKC - 1) / kStreamKC;
+    a.wide = K % 64 == 0;
     a.n_units = n_tiles * a.n_chunks;
     a.x_hi = x_hi;
     a.x_lo = x_lo;
@@ -481,7 +509,8 @@ int check_config(const ssd_config* c) {
     if (!(c->rms_eps > 0.f) || !(c->rope_theta > 0.f))
         return fail(SSD_ERR_INVALID_ARG, "rms_eps and rope_theta must be positive");
     const int G = c->n_heads / c->n_kv_heads;
-    if (attention_smem_bytes(c->head_dim, G, 8) > forward_smem_bytes(8) ||
+    if (attention_smem_bytes(c->head_dim, G, 1) > forward_smem_bytes(1) ||
+        attention_smem_bytes(c->head_dim, G, 8) > forward_smem_bytes(8) ||
         attention_smem_bytes(c->head_dim, G, kMaxRows) > forward_smem_bytes(kMaxRows))
         return fail(SSD_ERR_INVALID_ARG, "n_heads / n_kv_heads too large");
     return SSD_OK;
@@ -606,11 +635,11 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
     const size_t HD = c.head_dim;
     if ((rc = dalloc(h, &h->kc, h->kv_layer * L, &B)) || (rc = dalloc(h, &h->vc, h->kv_layer * L, &B)) ||
         (rc = dalloc(h, &h->h, (size_t)kMaxRows * d, &B)) ||
-        (rc = dalloc(h, &h->xn_hi, (size_t)kMaxRows * d, &B)) || (rc = dalloc(h, &h->xn_lo, (size_t)kMaxRows * d, &B)) ||
+        (rc = dalloc(h, &h->xn_hi, (size_t)2 * kMaxRows * d, &B)) ||
         (rc = dalloc(h, &h->ss, (size_t)kMaxRows * (d / kTileRows), &B)) ||
         (rc = dalloc(h, &h->q, (size_t)kMaxRows * qd, &B)) ||
-        (rc = dalloc(h, &h->at_hi, (size_t)kMaxRows * qd, &B)) || (rc = dalloc(h, &h->at_lo, (size_t)kMaxRows * qd, &B)) ||
-        (rc = dalloc(h, &h->ac_hi, (size_t)kMaxRows * F, &B)) || (rc = dalloc(h, &h->ac_lo, (size_t)kMaxRows * F, &B)) ||
+        (rc = dalloc(h, &h->at_hi, (size_t)2 * kMaxRows * qd, &B)) ||
+        (rc = dalloc(h, &h->ac_hi, (size_t)2 * kMaxRows * F, &B)) ||
         (rc = dalloc(h, &h->logits, (size_t)kMaxRows * V, &B)) ||
         (rc = dalloc(h, &h->p_rows, (size_t)kMaxRows * V, &B)) ||
         (rc = dalloc(h, &h->q_rows, (size_t)kMaxRows * V, &B)) || (rc = dalloc(h, &h->partial, part, &B)) ||
@@ -622,12 +651,17 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
         (rc = dalloc(h, &h->st, 1, &B)) || (rc = dalloc(h, &h->bar, 4, &B)))
         return bail(rc);
     h->max_ops = 2 + 5 * L;
-    h->n_tmaps = 7 * L + 1 + 18;
+    if (h->max_ops + 1 > 1024) return bail(fail(SSD_ERR_INVALID_ARG, "too many layers (at most 204)"));
+    h->n_tmaps = 7 * L + 1 + 9;
     if ((rc = dalloc(h, &h->tmaps, (size_t)h->n_tmaps, &B)) ||
         (rc = dalloc(h, &h->ops_full, (size_t)h->max_ops, &B)) ||
         (rc = dalloc(h, &h->ops_draft, (size_t)h->max_ops, &B)) ||
-        (rc = dalloc(h, &h->trace, (size_t)h->max_ops + 1, &B)))
+        (rc = dalloc(h, &h->trace, (size_t)1024 + 64 * 4, &B)))
         return bail(rc);
+    // the lo plane follows the hi plane: [2][16][K]
+    h->xn_lo = h->xn_hi + (size_t)kMaxRows * d;
+    h->at_lo = h->at_hi + (size_t)kMaxRows * qd;
+    h->ac_lo = h->ac_hi + (size_t)kMaxRows * F;
     {
         cudaError_t e = cudaMallocHost(&h->st_host, sizeof(DecodeState));
         if (e == cudaSuccess) e = cudaMallocHost(&h->emitted_host, sizeof(int) * 4);
@@ -828,14 +862,17 @@ int ssd_debug_forward(ssd_handle* h, int draft, const int32_t* tokens, int n_row
 }
 
 // Per-op durations (us) of one forward replay from the device trace.
-int trace_forward(ssd_handle* h, cudaGraphExec_t exec, int n_ops, std::vector<float>* us) {
-    std::vector<unsigned long long> t((size_t)n_ops + 1);
+int trace_forward(ssd_handle* h, cudaGraphExec_t exec, int n_ops, std::vector<float>* us,
+                  std::vector<unsigned long long>* units = nullptr) {
+    std::vector<unsigned long long> t(1024 + 64 * 4);
+    CUDA_TRY(cudaMemsetAsync(h->trace, 0, t.size() * sizeof(unsigned long long), h->stream), "trace reset");
     CUDA_TRY(cudaGraphLaunch(exec, h->stream), "traced replay");
     CUDA_TRY(cudaMemcpyAsync(t.data(), h->trace, t.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost,
                              h->stream), "trace read");
     CUDA_TRY(cudaStreamSynchronize(h->stream), "trace");
     us->resize(n_ops);
     for (int o = 0; o < n_ops; ++o) (*us)[o] = (float)((double)(t[o + 1] - t[o]) * 1e-3);
+    if (units) units->assign(t.begin() + 1024, t.end());
     return SSD_OK;
 }
 
@@ -913,7 +950,7 @@ int ssd_debug_time_forward(ssd_handle* h, int draft, int rows, int gemm_only, in
 }
 
 int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, int* op_types, int max_ops,
-                            int* n_ops_out) {
+                            int* n_ops_out, unsigned long long* unit_trace) {
     if (!h || !op_us || !op_types || !n_ops_out) return fail(SSD_ERR_INVALID_ARG, "NULL argument");
     if (rows < 1 || rows > kMaxRows || rows > h->cfg.max_seq) return fail(SSD_ERR_INVALID_ARG, "rows in [1, 16]");
     const int n_ops = draft ? h->n_ops_draft : h->n_ops_full;
@@ -924,8 +961,9 @@ int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, in
     int rc = capture_debug_forward(h, draft, rows, true, &traced, &n);
     if (rc) return rc;
     std::vector<float> us;
+    std::vector<unsigned long long> units;
     CUDA_TRY(cudaGraphLaunch(traced, h->stream), "warm-up");
-    rc = trace_forward(h, traced, n_ops, &us);
+    rc = trace_forward(h, traced, n_ops, &us, &units);
     cudaGraphExecDestroy(traced);
     if (rc) return rc;
     std::vector<FwdOp> ops = build_ops(h, draft != 0);
@@ -933,6 +971,7 @@ int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, in
         op_us[o] = us[o];
         op_types[o] = ops[o].type;
     }
+    if (unit_trace) for (size_t i = 0; i < units.size(); ++i) unit_trace[i] = units[i];
     *n_ops_out = n_ops;
     return SSD_OK;
 }

@@ -170,54 +170,96 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, int x, 
         : "memory");
 }
 
+__device__ __forceinline__ void tma_load_4d(void* dst, const void* tmap, int x, int y, int z, int w, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];"
+        ::"r"(smem_u32(dst)), "l"(tmap), "r"(x), "r"(y), "r"(z), "r"(w), "r"(smem_u32(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_3d(void* dst, const void* tmap, int x, int y, int z, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
+        ::"r"(smem_u32(dst)), "l"(tmap), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+        : "memory");
+}
+
 // ---------------------------------------------------------------------------
 // projection op
 // ---------------------------------------------------------------------------
-// Stage layout (every box 1 KB aligned, 128-byte swizzle: 16-byte chunk c of
-// row r sits at chunk c ^ (r & 7)):
-//   weights: 4 k-boxes x 64 rows x 128 B  (k-box stride 8 KB; rows 0-31 and
-//            32-63 are two TMA boxes of 4 KB)
-//   inputs : 4 k-boxes x (P hi rows + P lo rows) x 128 B
-template <int P>
+// Stage layout (1 KB aligned boxes; 128-byte swizzle: 16-byte chunk c of a
+// 128-byte smem row at address A sits at chunk c ^ ((A >> 7) & 7)).
+// wide layout (K % 64 == 0):
+//   weights: [half 2][row 32][k-box 4][64 bf16]: row r of the tile at
+//            (r >> 5) * 16 KB + (r & 31) * 512 + kbox * 128
+//   inputs : [plane 2][row R][k-box 4][64 bf16]: MMA row p = plane * R + row at
+//            p * 512 + kbox * 128 (rows past 2R only feed unused output columns)
+// narrow layout (K % 64 != 0, one copy per 64-wide k-box):
+//   weights: [k-box 4][row 64][64]: kbox * 8 KB + r * 128
+//   inputs : [k-box 4][max(2R, 8) rows][64]: kbox * XKB + p * 128
+template <int R>
 struct GemmSmem {
-    static constexpr int WB = kTileRows * ROWB;         // 32 KB
-    static constexpr int XKB = 2 * P * 128;             // input bytes per k-box
-    static constexpr int XB = 4 * XKB;
+    static constexpr int NT = (2 * R + 7) / 8;   // n8 MMA tiles: 1 | 2 | 4
+    static constexpr int XR = NT * 8;            // input rows the MMA reads
+    static constexpr int WB = kTileRows * ROWB;  // 32 KB
+    static constexpr int XKB = XR * 128;         // narrow layout: input bytes per k-box
+    static constexpr int XB = XR * ROWB;         // = 4 * XKB
     static constexpr int STAGE = WB + XB;
-    static constexpr int RC = 2 * P;
+    static constexpr int RC = NT * 8;
     static constexpr size_t BYTES = 1024 + (size_t)S * STAGE + kTileRows * RC * 4 + kTileRows * 16 * 4;
 };
 
-__device__ __forceinline__ int x_class(int M) { return M == 1 ? 0 : (M <= 8 ? 1 : 2); }
-__device__ __forceinline__ int x_rows(int M) { return M == 1 ? 1 : (M <= 8 ? 8 : 16); }
+// byte offset of 16-byte chunk c (0..7) of k-box kb in row r of the weights,
+// or row p of the inputs (the swizzle XOR follows the address)
+__device__ __forceinline__ int w_off(bool wide, int r, int kb, int c) {
+    if (wide) {
+        const int a = (r >> 5) * 16384 + (r & 31) * 512 + kb * 128;
+        return a + ((c ^ ((a >> 7) & 7)) << 4);
+    }
+    const int a = kb * 8192 + r * 128;
+    return a + ((c ^ (r & 7)) << 4);
+}
+template <int R>
+__device__ __forceinline__ int x_off(bool wide, int p, int kb, int c) {
+    if (wide) {
+        const int a = p * 512 + kb * 128;
+        return a + ((c ^ ((a >> 7) & 7)) << 4);
+    }
+    const int a = kb * GemmSmem<R>::XKB + p * 128;
+    return a + ((c ^ (p & 7)) << 4);
+}
 
-// the two 32-row TMA boxes of a 64-row tile: (map, first row) for rows 0-31 and 32-63
-__device__ __forceinline__ void tile_boxes(const GemmArgs& a, int epi, int tile, const void** m0, int* r0,
-                                           const void** m1, int* r1) {
+// Sources of a 64-row tile as two 32-row halves: rows r0.. of map m0, then
+// rows r1.. of map m1.  Halves come from two places for the RoPE pairs of q /
+// k (rotation partners j and j + head_dim/2) and for gate + up.
+__device__ __forceinline__ void tile_halves(const GemmArgs& a, int epi, int tile, const void** m0, int* r0,
+                                            const void** m1, int* r1) {
     if (epi == EPI_LOGITS || epi == EPI_RESID) {
         *m0 = *m1 = a.tm_w[0];
         *r0 = tile * kTileRows;
         *r1 = *r0 + 32;
-    } else if (epi == EPI_SWIGLU) {  // gate rows, up rows
+        return;
+    }
+    if (epi == EPI_SWIGLU) {  // gate rows, up rows
         *m0 = a.tm_w[0];
         *m1 = a.tm_w[1];
         *r0 = *r1 = tile * 32;
-    } else {  // QKV: q / k tiles hold RoPE pairs (i, i + hd/2); v tiles are plain
-        const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
-        const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
-        if (tile < q_tiles + k_tiles) {
-            const bool is_q = tile < q_tiles;
-            const int tt = is_q ? tile : tile - q_tiles;
-            const int head = tt / per_head, j0 = (tt % per_head) * 32;
-            *m0 = *m1 = is_q ? a.tm_w[0] : a.tm_w[1];
-            *r0 = head * hd + j0;
-            *r1 = head * hd + half + j0;
-        } else {
-            *m0 = *m1 = a.tm_w[2];
-            *r0 = (tile - q_tiles - k_tiles) * kTileRows;
-            *r1 = *r0 + 32;
-        }
+        return;
     }
+    const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
+    const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
+    if (tile < q_tiles + k_tiles) {
+        const bool is_q = tile < q_tiles;
+        const int tt = is_q ? tile : tile - q_tiles;
+        const int head = tt / per_head, j0 = (tt % per_head) * 32;
+        *m0 = *m1 = is_q ? a.tm_w[0] : a.tm_w[1];
+        *r0 = head * hd + j0;
+        *r1 = head * hd + half + j0;
+        return;
+    }
+    *m0 = *m1 = a.tm_w[2];
+    *r0 = (tile - q_tiles - k_tiles) * kTileRows;
+    *r1 = *r0 + 32;
 }
 
 __device__ __forceinline__ int unit_kboxes(const GemmArgs& a, int u) {
@@ -225,33 +267,43 @@ __device__ __forceinline__ int unit_kboxes(const GemmArgs& a, int u) {
     return min(4, (a.K - k0 + 63) / 64);
 }
 
-// weights of unit u into a stage (one thread): expect_tx without arriving
-template <int P>
+// weights of unit u into a stage (one thread): expect_tx without arriving.
+// Bytes are always a full 64 x 256 tile (out-of-range rows / columns are
+// delivered as zeros and counted).
+template <int R>
 __device__ __forceinline__ void tma_weights(const GemmArgs& a, int epi, int u, unsigned char* st, uint64_t* bar) {
     const int tile = u / a.n_chunks, k0 = (u - tile * a.n_chunks) * KC;
-    const int nkb = unit_kboxes(a, u);
     const void *m0, *m1;
     int r0, r1;
-    tile_boxes(a, epi, tile, &m0, &r0, &m1, &r1);
-    mbar_expect_tx(bar, (unsigned)nkb * 2u * 32u * 128u);
-    for (int kb = 0; kb < nkb; ++kb) {
-        tma_load_2d(st + kb * 8192, m0, k0 + kb * 64, r0, bar);
-        tma_load_2d(st + kb * 8192 + 4096, m1, k0 + kb * 64, r1, bar);
+    tile_halves(a, epi, tile, &m0, &r0, &m1, &r1);
+    if (a.wide) {
+        mbar_expect_tx(bar, 32768u);
+        tma_load_3d(st, m0, 0, k0 >> 6, r0, bar);
+        tma_load_3d(st + 16384, m1, 0, k0 >> 6, r1, bar);
+    } else {
+        const int nkb = unit_kboxes(a, u);
+        mbar_expect_tx(bar, (unsigned)nkb * 8192u);
+        for (int kb = 0; kb < nkb; ++kb) {
+            tma_load_2d(st + kb * 8192, m0, k0 + kb * 64, r0, bar);
+            tma_load_2d(st + kb * 8192 + 4096, m1, k0 + kb * 64, r1, bar);
+        }
     }
 }
 
 // input planes of unit u into a stage (one thread): arrive + expect_tx
-template <int P>
-__device__ __forceinline__ void tma_inputs(const GemmArgs& a, int M, int u, unsigned char* st, uint64_t* bar) {
-    using L = GemmSmem<P>;
+template <int R>
+__device__ __forceinline__ void tma_inputs(const GemmArgs& a, int u, unsigned char* st, uint64_t* bar) {
+    using L = GemmSmem<R>;
     const int k0 = (u % a.n_chunks) * KC;
-    const int nkb = unit_kboxes(a, u);
-    const int cls = x_class(M), rows = x_rows(M);
-    mbar_arrive_expect_tx(bar, (unsigned)nkb * 2u * (unsigned)rows * 128u);
+    const int cls = R == 1 ? 0 : (R == 8 ? 1 : 2);
     unsigned char* xs = st + L::WB;
-    for (int kb = 0; kb < nkb; ++kb) {
-        tma_load_2d(xs + kb * L::XKB, a.tm_x[cls][0], k0 + kb * 64, 0, bar);
-        tma_load_2d(xs + kb * L::XKB + P * 128, a.tm_x[cls][1], k0 + kb * 64, 0, bar);
+    if (a.wide) {
+        mbar_arrive_expect_tx(bar, 4u * 2u * (unsigned)R * 128u);
+        tma_load_4d(xs, a.tm_x[cls], 0, k0 >> 6, 0, 0, bar);
+    } else {
+        const int nkb = unit_kboxes(a, u);
+        mbar_arrive_expect_tx(bar, (unsigned)nkb * 2u * (unsigned)R * 128u);
+        for (int kb = 0; kb < nkb; ++kb) tma_load_3d(xs + kb * L::XKB, a.tm_x[cls], k0 + kb * 64, 0, 0, bar);
     }
 }
 
@@ -267,7 +319,7 @@ struct Pipe {
 
 // Producer: requests the weights of this CTA's first S units of a projection
 // before the grid barrier (they do not depend on the previous op).
-template <int P>
+template <int R>
 __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, Pipe& pp, int* err) {
     int u_begin, n_my;
     my_units(a.n_units, &u_begin, &n_my);
@@ -276,7 +328,7 @@ __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, P
         for (int s = 0; s < S && s < n_my; ++s) {
             if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return false;
             pp.pphase ^= 1u << s;
-            tma_weights<P>(a, epi, u_begin + s, smem + s * GemmSmem<P>::STAGE, pp.full + s);
+            tma_weights<R>(a, epi, u_begin + s, smem + s * GemmSmem<R>::STAGE, pp.full + s);
         }
     }
     return true;
@@ -285,11 +337,13 @@ __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, P
 // Returns false if a TMA wait timed out (error recorded).  The producer warp
 // (one elected thread) streams this CTA's units through the S stages; the 8
 // consumer warps compute and release each stage with one arrival per warp.
-template <int P>
+// ut: nullptr, or [64][4] timestamps of this CTA's first units (producer
+// issue, consumer data ready, MMA done, flush done) - a profiling aid.
+template <int R>
 __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefetched, unsigned char* smem,
-                        float* r_s, Pipe& pp, int* err) {
-    using L = GemmSmem<P>;
-    constexpr int NT = 2 * (P / 8), RC = L::RC;
+                        float* r_s, Pipe& pp, int* err, unsigned long long* ut) {
+    using L = GemmSmem<R>;
+    constexpr int NT = L::NT, RC = L::RC;
     float* red = reinterpret_cast<float*>(smem + S * L::STAGE);  // [64][RC]
     float* ys = red + kTileRows * RC;                             // [64][16]
     __shared__ int s_last;
@@ -305,12 +359,13 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         for (int i = 0; i < n_my; ++i) {
             const int s = i % S;
             unsigned char* st = smem + s * L::STAGE;
+            if (ut && i < 64) ut[i * 4 + 0] = globaltimer();
             if (!(prefetched && i < S)) {
                 if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return false;
                 pp.pphase ^= 1u << s;
-                tma_weights<P>(a, epi, u_begin + i, st, pp.full + s);
+                tma_weights<R>(a, epi, u_begin + i, st, pp.full + s);
             }
-            tma_inputs<P>(a, M, u_begin + i, st, pp.full + s);
+            tma_inputs<R>(a, u_begin + i, st, pp.full + s);
         }
         return true;
     }
@@ -345,21 +400,21 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         const unsigned char* x_s = w_s + L::WB;
         if (!mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err)) return false;
         pp.cphase ^= 1u << s;
+        if (ut && i < 64 && threadIdx.x == 0) ut[i * 4 + 1] = globaltimer();
 
-        // k32 block kb: k-box kb/2; thread tig reads 16-byte chunk 2*tig + (kb & 1)
-        // of its rows (A: weight rows r0, r0 + 8; B: input rows nt*8 + g); both
-        // operands use the same chunk -> logical-k mapping.  Columns past K are
-        // zero-filled by TMA in both operands.
+        // A: weight rows r0, r0 + 8; B: input rows nt*8 + g.  Both operands use
+        // the same chunk -> logical-k mapping, so the product is unchanged;
+        // columns past K are zero-filled by TMA in both operands.
         const int nb = (kc_eff + 31) >> 5;
+        const bool wide = a.wide != 0;
         auto block = [&](int kb, float (&ac)[NT][4]) {
-            const int ch = ((2 * tig + (kb & 1)) ^ g) * 16;
-            const unsigned char* wk = w_s + (kb >> 1) * 8192;
-            const unsigned char* xk = x_s + (kb >> 1) * L::XKB;
-            const uint4 wa = *reinterpret_cast<const uint4*>(wk + r0 * 128 + ch);
-            const uint4 wb = *reinterpret_cast<const uint4*>(wk + (r0 + 8) * 128 + ch);
+            // k32 block kb = 16-byte chunks 4*(kb&1) .. +3 of k-box kb/2; thread tig takes chunk 4*(kb&1) + tig
+            const int kbx = kb >> 1, c = 4 * (kb & 1) + tig;
+            const uint4 wa = *reinterpret_cast<const uint4*>(w_s + w_off(wide, r0, kbx, c));
+            const uint4 wb = *reinterpret_cast<const uint4*>(w_s + w_off(wide, r0 + 8, kbx, c));
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
-                const uint4 xv = *reinterpret_cast<const uint4*>(xk + (nt * 8 + g) * 128 + ch);
+                const uint4 xv = *reinterpret_cast<const uint4*>(x_s + x_off<R>(wide, nt * 8 + g, kbx, c));
                 mma_bf16_16816(ac[nt], wa.x, wb.x, wa.y, wb.y, xv.x, xv.y);
                 mma_bf16_16816(ac[nt], wa.z, wb.z, wa.w, wb.w, xv.z, xv.w);
             }
@@ -370,6 +425,7 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(pp.empty + s);  // this warp is done with the stage
+        if (ut && i < 64 && threadIdx.x == 0) ut[i * 4 + 2] = globaltimer();
 
         if (!(i == n_my - 1 || chunk == a.n_chunks - 1)) continue;
 
@@ -408,7 +464,7 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         consumer_sync();
         for (int idx = threadIdx.x; idx < kTileRows * M; idx += kGemmThreads) {
             const int m = idx / kTileRows, r = idx - m * kTileRows;
-            ys[r * 16 + m] = red[r * RC + m] + red[r * RC + P + m];
+            ys[r * 16 + m] = red[r * RC + m] + red[r * RC + R + m];
         }
         consumer_sync();
 
@@ -522,6 +578,7 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
             }
         }
         consumer_sync();  // ys / red are reused by the next segment
+        if (ut && i < 64 && threadIdx.x == 0) ut[i * 4 + 3] = globaltimer();
     }
     consumer_sync();
     return true;
@@ -733,7 +790,7 @@ __device__ void drain_before_exit() {
     __syncthreads();
 }
 
-template <int NPH, int HD>
+template <int R, int HD>
 __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams p) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     __shared__ float r_s[kMaxRows];
@@ -741,7 +798,6 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
     __shared__ __align__(8) uint64_t full[S];   // TMA completion per stage
     __shared__ __align__(8) uint64_t empty[S];  // stage released by the 8 consumer warps
     __shared__ FwdOp s_op[2];                   // current and next op's arguments
-    constexpr int P = 8 * NPH;
     // 128-byte TMA swizzle needs 1 KB aligned boxes
     unsigned char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     if (threadIdx.x == 0) {
@@ -774,13 +830,15 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         bool ok = true;
         if (type == OP_EMBED) embed_op(p, pos0);
         else if (type == OP_ATTN) attn_op<HD>(op.at, p.M, pos0, smem);
-        else ok = gemm_op<P>(op.g, epi_of(type), p.M, pos0, prefetched, smem, r_s, pp, p.err);
+        else
+            ok = gemm_op<R>(op.g, epi_of(type), p.M, pos0, prefetched, smem, r_s, pp, p.err,
+                            (p.trace && blockIdx.x == 0 && o == 1) ? p.trace + 1024 : nullptr);
         prefetched = false;
         if (o + 1 < p.n_ops) {
             copy_op(p.ops + o + 1, s_op + ((o + 1) & 1));  // (all threads, includes a barrier)
             const FwdOp& nx = s_op[(o + 1) & 1];
             if (ok && is_gemm(nx.type)) {
-                ok = gemm_prefetch<P>(nx.g, epi_of(nx.type), smem, pp, p.err);
+                ok = gemm_prefetch<R>(nx.g, epi_of(nx.type), smem, pp, p.err);
                 prefetched = true;
             }
         }
@@ -801,30 +859,33 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
     }
 }
 
-template <int NPH, int HD>
+template <int R, int HD>
 int launch_fwd(const FwdParams& p, int grid, cudaStream_t s) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid, 1, 1);
     cfg.blockDim = dim3(kFwdThreads, 1, 1);
-    cfg.dynamicSmemBytes = GemmSmem<8 * NPH>::BYTES;
+    cfg.dynamicSmemBytes = GemmSmem<R>::BYTES;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeCooperative;
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return (int)cudaLaunchKernelEx(&cfg, forward_kernel<NPH, HD>, p);
+    return (int)cudaLaunchKernelEx(&cfg, forward_kernel<R, HD>, p);
 }
 
-template <int NPH, int HD>
+template <int R, int HD>
 int configure_fwd() {
-    return (int)cudaFuncSetAttribute(forward_kernel<NPH, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)GemmSmem<8 * NPH>::BYTES);
+    return (int)cudaFuncSetAttribute(forward_kernel<R, HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)GemmSmem<R>::BYTES);
 }
 
 }  // namespace
 
-size_t forward_smem_bytes(int M) { return M <= 8 ? GemmSmem<8>::BYTES : GemmSmem<16>::BYTES; }
+size_t forward_smem_bytes(int M) {
+    const int R = fwd_plane_rows(M);
+    return R == 1 ? GemmSmem<1>::BYTES : (R == 8 ? GemmSmem<8>::BYTES : GemmSmem<16>::BYTES);
+}
 
 size_t attention_smem_bytes(int head_dim, int group, int M) {
     return 2 * kAttnChunk * (head_dim * 2 + 16) + (size_t)group * M * head_dim * 4 + 8 * kAttnChunk * 4;
@@ -833,16 +894,20 @@ size_t attention_smem_bytes(int head_dim, int group, int M) {
 int forward_configure() {
     int e = 0;
     e = e ? e : configure_fwd<1, 64>();
-    e = e ? e : configure_fwd<2, 64>();
+    e = e ? e : configure_fwd<8, 64>();
+    e = e ? e : configure_fwd<16, 64>();
     e = e ? e : configure_fwd<1, 128>();
-    e = e ? e : configure_fwd<2, 128>();
+    e = e ? e : configure_fwd<8, 128>();
+    e = e ? e : configure_fwd<16, 128>();
     return e;
 }
 
 int launch_forward(const FwdParams& p, int head_dim, int grid, cudaStream_t s) {
-    const bool two = p.M > 8;
-    if (head_dim == 128) return two ? launch_fwd<2, 128>(p, grid, s) : launch_fwd<1, 128>(p, grid, s);
-    if (head_dim == 64) return two ? launch_fwd<2, 64>(p, grid, s) : launch_fwd<1, 64>(p, grid, s);
+    const int R = fwd_plane_rows(p.M);
+    if (head_dim == 128)
+        return R == 1 ? launch_fwd<1, 128>(p, grid, s) : (R == 8 ? launch_fwd<8, 128>(p, grid, s) : launch_fwd<16, 128>(p, grid, s));
+    if (head_dim == 64)
+        return R == 1 ? launch_fwd<1, 64>(p, grid, s) : (R == 8 ? launch_fwd<8, 64>(p, grid, s) : launch_fwd<16, 64>(p, grid, s));
     return (int)cudaErrorInvalidValue;
 }
 

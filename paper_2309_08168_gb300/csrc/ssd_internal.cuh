@@ -82,8 +82,15 @@ struct GemmArgs {
     float* ss_out;       // EPI_RESID: [M][n_tiles] per-tile sums of h^2
     int n_chunks;        // ceil(K / kStreamKC)
     int n_units;         // n_tiles * n_chunks
-    const void* tm_w[3];     // TMA tensor maps (global memory) of w0, w1, w2: box 64 k x 32 rows
-    const void* tm_x[3][2];  // TMA maps of the input planes [box rows 1 | 8 | 16][hi | lo]
+    // TMA tensor maps (in global memory).  wide = 1 (K % 64 == 0): w maps view
+    // W as {64, K/64, rows} with box {64, 4, 32} (one copy per 32-row half of
+    // a unit), x maps view the planes as {64, K/64, 16, 2} with box
+    // {64, 4, R, 2} (one copy per unit).  wide = 0: 2D w maps with box
+    // {64, 32} and 3D x maps {64, 16, 2} with box {64, R, 2}, one copy per
+    // 64-wide k-box.
+    int wide;
+    const void* tm_w[3];  // w0, w1, w2
+    const void* tm_x[3];  // input planes for R = 1 | 8 | 16
 };
 
 // ---------------------------------------------------------------------------
@@ -150,6 +157,7 @@ int gemm_configure();
 int launch_gemm(int epi, const GemmArgs& a, cudaStream_t s);
 size_t gemm_smem_bytes(int kc, int M);
 constexpr int gemm_half_rows(int M) { return M <= 8 ? 8 : 16; }  // padded rows of x_hi (and of x_lo)
+constexpr int fwd_plane_rows(int M) { return M == 1 ? 1 : (M <= 8 ? 8 : 16); }  // R of the forward kernel
 
 
 
