@@ -174,12 +174,18 @@ int ssd_debug_time_forward(ssd_handle* h, int draft, int rows, int gemm_only, in
  * of op o-1 to the end of op o, grid barrier included), op_types[o] = 0
  * embedding, 1 q/k/v projection, 2 attention, 3 output or down projection,
  * 4 gate/up projection, 5 lm_head.  max_ops >= 2 + 5 * n_layers is always
- * enough.  unit_trace (may be NULL): 256 globaltimer stamps (ns) of CTA 0's
- * first 64 work units of the first projection, 4 per unit: producer issue,
- * consumer data ready, MMA done, segment flush done (0 if none).
+ * enough.  detail_op: index of one op to trace in detail (-1: none).
+ * unit_trace (may be NULL): 256 globaltimer stamps (ns) of CTA 0's first 64
+ * work units of detail_op when it is a projection, 4 per unit: producer
+ * issue, consumer data ready, MMA done, segment flush done (0 if none).
+ * cta_trace (may be NULL): 8 stamps per CTA of the forward kernel for
+ * detail_op: op start, first data ready, last MMA done, work done, grid
+ * barrier arrive, barrier release, number of work units, 0; max_ctas >= the
+ * grid (the SM count), *n_ctas = the grid.
  * Errors: INVALID_ARG, CUDA. */
 int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, int* op_types,
-                            int max_ops, int* n_ops, unsigned long long* unit_trace);
+                            int max_ops, int* n_ops, int detail_op, unsigned long long* unit_trace,
+                            unsigned long long* cta_trace, int max_ctas, int* n_ctas);
 
 /* Allocation-free projection.  The paper has no counterpart: this is a
  * service of this library for callers that cannot allocate device memory

@@ -82,7 +82,8 @@ def _load():
     lib.ssd_debug_spec_accept.argtypes = [H, _VP, _VP, ctypes.c_int, _VP, _VP, ctypes.c_int, ctypes.c_int, _VP]
     lib.ssd_debug_time_forward.argtypes = [H, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                            _VP, _VP, _VP]
-    lib.ssd_debug_trace_forward.argtypes = [H, ctypes.c_int, ctypes.c_int, _VP, _VP, ctypes.c_int, _VP, _VP]
+    lib.ssd_debug_trace_forward.argtypes = [H, ctypes.c_int, ctypes.c_int, _VP, _VP, ctypes.c_int, _VP,
+                                            ctypes.c_int, _VP, _VP, ctypes.c_int, _VP]
     lib.ssd_debug_trace_forward.restype = ctypes.c_int
     lib.ssd_linear_noalloc.argtypes = [_VP, _VP, _VP, ctypes.c_int, ctypes.c_int, ctypes.c_int, _VP]
     lib.ssd_linear_noalloc.restype = ctypes.c_int
@@ -186,20 +187,28 @@ def ssd_linear_noalloc(w, x, y, N: int, K: int, M: int, cuda_stream: int | None 
 OP_NAMES = ("embed", "qkv", "attention", "o/down", "gate/up", "lm_head")
 
 
-def ssd_debug_trace_forward(h: int, draft: bool, rows: int, units: bool = False):
-    """Returns [(op name, microseconds)] for one forward of the forward kernel
-    (and, with units=True, also the [64][4] unit stamps of CTA 0's first
-    projection, in ns)."""
+def ssd_debug_trace_forward(h: int, draft: bool, rows: int, detail_op: int = -1):
+    """Returns [(op name, microseconds)] for one forward of the forward kernel.
+    With detail_op >= 0 it returns (ops, units, ctas): units = [64][4] stamps
+    (ns) of CTA 0's first work units of that op (producer issue, data ready,
+    MMA done, flush done), ctas = [grid][8] stamps per CTA (op start, first
+    data ready, last MMA done, work done, barrier arrive, barrier release,
+    units, 0)."""
     cfg = config_of(h)
     cap = 2 + 5 * cfg.n_layers
     us = np.zeros(cap, dtype=np.float32)
     ty = np.zeros(cap, dtype=np.int32)
     ut = np.zeros((64, 4), dtype=np.uint64)
+    max_ctas = 1024
+    ct = np.zeros((max_ctas, 8), dtype=np.uint64)
     n = ctypes.c_int()
+    n_ctas = ctypes.c_int()
+    detail = detail_op >= 0
     _check(lib.ssd_debug_trace_forward(h, int(draft), rows, us.ctypes.data, ty.ctypes.data, cap,
-                                       ctypes.addressof(n), ut.ctypes.data))
+                                       ctypes.addressof(n), int(detail_op), ut.ctypes.data if detail else None,
+                                       ct.ctypes.data if detail else None, max_ctas, ctypes.addressof(n_ctas)))
     ops = [(OP_NAMES[ty[i]], float(us[i])) for i in range(n.value)]
-    return (ops, ut) if units else ops
+    return (ops, ut, ct[:n_ctas.value]) if detail else ops
 
 
 def ssd_destroy(h: int) -> None:
@@ -286,5 +295,5 @@ class Decoder:
     def debug_time_forward(self, draft, rows, gemm_only, reps):
         return ssd_debug_time_forward(self.h, draft, rows, gemm_only, reps)
 
-    def debug_trace_forward(self, draft, rows, units=False):
-        return ssd_debug_trace_forward(self.h, draft, rows, units)
+    def debug_trace_forward(self, draft, rows, detail_op=-1):
+        return ssd_debug_trace_forward(self.h, draft, rows, detail_op)

@@ -113,7 +113,8 @@ struct ssd_handle {
     bf16* ac_lo = nullptr;
     int n_sms = 0;
     unsigned* bar = nullptr;            // grid-barrier counter of the forward kernel
-    unsigned long long* trace = nullptr;  // per-op timestamps (profiling hook)
+    unsigned long long* trace = nullptr;  // per-op timestamps (profiling hook, FwdParams::trace)
+    int trace_op = -1;                    // op traced per unit and per CTA
     CUtensorMap* tmaps = nullptr;       // TMA descriptors (weights, input planes) in device memory
     int n_tmaps = 0;
     FwdOp* ops_full = nullptr;          // op lists in device memory
@@ -178,6 +179,8 @@ const bf16* next_norm(const ssd_handle* h, int s, bool draft) {
 // with buf 0 = normalised rows (K = d), 1 = attention output (K = H*hd),
 // 2 = SwiGLU output (K = ffn) and cls = rows per plane 1 | 8 | 16.
 // ---------------------------------------------------------------------------
+size_t trace_words(const ssd_handle* h) { return (size_t)kTraceCtas + 8 * (size_t)h->n_sms; }
+
 int tmap_weight(int l, int which) { return 7 * l + which; }
 int tmap_x(const ssd_handle* h, int buf, int cls) { return 7 * h->cfg.n_layers + 1 + buf * 3 + cls; }
 
@@ -404,6 +407,7 @@ int forward(ssd_handle* h, int M, int src, const int* toks, int pos0, bool draft
     p.bar = h->bar;
     p.err = &h->st->err;
     p.trace = trace;
+    p.trace_op = h->trace_op;
     CUDA_TRY(cudaMemsetAsync(h->bar, 0, sizeof(unsigned), h->stream), "barrier reset");
     LAUNCH(h, launch_forward(p, c.head_dim, h->n_sms, h->stream), "forward kernel", -1);
     if (n_launch) *n_launch = 1;
@@ -656,7 +660,7 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
     if ((rc = dalloc(h, &h->tmaps, (size_t)h->n_tmaps, &B)) ||
         (rc = dalloc(h, &h->ops_full, (size_t)h->max_ops, &B)) ||
         (rc = dalloc(h, &h->ops_draft, (size_t)h->max_ops, &B)) ||
-        (rc = dalloc(h, &h->trace, (size_t)1024 + 64 * 4, &B)))
+        (rc = dalloc(h, &h->trace, trace_words(h), &B)))
         return bail(rc);
     // the lo plane follows the hi plane: [2][16][K]
     h->xn_lo = h->xn_hi + (size_t)kMaxRows * d;
@@ -861,10 +865,11 @@ int ssd_debug_forward(ssd_handle* h, int draft, const int32_t* tokens, int n_row
     return SSD_OK;
 }
 
-// Per-op durations (us) of one forward replay from the device trace.
+// Per-op durations (us) of one forward replay from the device trace; units:
+// the rest of the trace (unit and CTA stamps of h->trace_op).
 int trace_forward(ssd_handle* h, cudaGraphExec_t exec, int n_ops, std::vector<float>* us,
                   std::vector<unsigned long long>* units = nullptr) {
-    std::vector<unsigned long long> t(1024 + 64 * 4);
+    std::vector<unsigned long long> t(trace_words(h));
     CUDA_TRY(cudaMemsetAsync(h->trace, 0, t.size() * sizeof(unsigned long long), h->stream), "trace reset");
     CUDA_TRY(cudaGraphLaunch(exec, h->stream), "traced replay");
     CUDA_TRY(cudaMemcpyAsync(t.data(), h->trace, t.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost,
@@ -872,7 +877,7 @@ int trace_forward(ssd_handle* h, cudaGraphExec_t exec, int n_ops, std::vector<fl
     CUDA_TRY(cudaStreamSynchronize(h->stream), "trace");
     us->resize(n_ops);
     for (int o = 0; o < n_ops; ++o) (*us)[o] = (float)((double)(t[o + 1] - t[o]) * 1e-3);
-    if (units) units->assign(t.begin() + 1024, t.end());
+    if (units) *units = t;
     return SSD_OK;
 }
 
@@ -950,15 +955,19 @@ int ssd_debug_time_forward(ssd_handle* h, int draft, int rows, int gemm_only, in
 }
 
 int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, int* op_types, int max_ops,
-                            int* n_ops_out, unsigned long long* unit_trace) {
+                            int* n_ops_out, int detail_op, unsigned long long* unit_trace,
+                            unsigned long long* cta_trace, int max_ctas, int* n_ctas) {
     if (!h || !op_us || !op_types || !n_ops_out) return fail(SSD_ERR_INVALID_ARG, "NULL argument");
     if (rows < 1 || rows > kMaxRows || rows > h->cfg.max_seq) return fail(SSD_ERR_INVALID_ARG, "rows in [1, 16]");
     const int n_ops = draft ? h->n_ops_draft : h->n_ops_full;
     if (max_ops < n_ops) return fail(SSD_ERR_INVALID_ARG, "max_ops smaller than the op list");
     CUDA_TRY(cudaSetDevice(h->device), "set device");
+    if (cta_trace && (!n_ctas || max_ctas < h->n_sms)) return fail(SSD_ERR_INVALID_ARG, "max_ctas below the grid");
     cudaGraphExec_t traced = nullptr;
     int n = 0;
+    h->trace_op = detail_op;
     int rc = capture_debug_forward(h, draft, rows, true, &traced, &n);
+    h->trace_op = -1;
     if (rc) return rc;
     std::vector<float> us;
     std::vector<unsigned long long> units;
@@ -971,7 +980,11 @@ int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, in
         op_us[o] = us[o];
         op_types[o] = ops[o].type;
     }
-    if (unit_trace) for (size_t i = 0; i < units.size(); ++i) unit_trace[i] = units[i];
+    if (unit_trace) for (int i = 0; i < kTraceCtas - kTraceUnits; ++i) unit_trace[i] = units[kTraceUnits + i];
+    if (cta_trace) {
+        for (int i = 0; i < 8 * h->n_sms; ++i) cta_trace[i] = units[kTraceCtas + i];
+        *n_ctas = h->n_sms;
+    }
     *n_ops_out = n_ops;
     return SSD_OK;
 }

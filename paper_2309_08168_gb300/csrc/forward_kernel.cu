@@ -44,7 +44,6 @@ namespace ssd {
 namespace {
 
 constexpr int KC = kStreamKC;
-constexpr int S = kStreamStages;
 constexpr int ROWB = KC * 2;  // bytes of one 64-row tile row of a unit
 constexpr unsigned long long kBarrierTimeoutNs = 2000000000ull;
 // 8 consumer warps (MMA, epilogues, attention, embedding) + 1 producer warp (TMA)
@@ -184,6 +183,11 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const void* tmap, int x, 
         : "memory");
 }
 
+// brings a tensor map descriptor (global memory) into the descriptor cache
+__device__ __forceinline__ void prefetch_tmap(const void* tmap) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(tmap) : "memory");
+}
+
 // ---------------------------------------------------------------------------
 // projection op
 // ---------------------------------------------------------------------------
@@ -206,6 +210,7 @@ struct GemmSmem {
     static constexpr int XB = XR * ROWB;         // = 4 * XKB
     static constexpr int STAGE = WB + XB;
     static constexpr int RC = NT * 8;
+    static constexpr int S = 4;  // ring depth (5 or 6 stages, where they fit, measured no faster)
     static constexpr size_t BYTES = 1024 + (size_t)S * STAGE + kTileRows * RC * 4 + kTileRows * 16 * 4;
 };
 
@@ -229,37 +234,27 @@ __device__ __forceinline__ int x_off(bool wide, int p, int kb, int c) {
     return a + ((c ^ (p & 7)) << 4);
 }
 
-// Sources of a 64-row tile as two 32-row halves: rows r0.. of map m0, then
-// rows r1.. of map m1.  Halves come from two places for the RoPE pairs of q /
-// k (rotation partners j and j + head_dim/2) and for gate + up.
-__device__ __forceinline__ void tile_halves(const GemmArgs& a, int epi, int tile, const void** m0, int* r0,
-                                            const void** m1, int* r1) {
-    if (epi == EPI_LOGITS || epi == EPI_RESID) {
-        *m0 = *m1 = a.tm_w[0];
-        *r0 = tile * kTileRows;
-        *r1 = *r0 + 32;
-        return;
-    }
-    if (epi == EPI_SWIGLU) {  // gate rows, up rows
-        *m0 = a.tm_w[0];
-        *m1 = a.tm_w[1];
-        *r0 = *r1 = tile * 32;
-        return;
-    }
+// Sources of a 64-row tile as two 32-row halves: rows r0.. of matrix s0, then
+// rows r1.. of matrix s1 (0, 1, 2 = w0, w1, w2).  Halves come from two places
+// for the RoPE pairs of q / k (rotation partners j and j + head_dim/2) and for
+// gate + up.
+struct Halves {
+    int s0, r0, s1, r1;
+};
+__device__ __forceinline__ Halves tile_halves(const GemmArgs& a, int epi, int tile) {
+    if (epi == EPI_LOGITS || epi == EPI_RESID) return {0, tile * kTileRows, 0, tile * kTileRows + 32};
+    if (epi == EPI_SWIGLU) return {0, tile * 32, 1, tile * 32};  // gate rows, up rows
     const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
     const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
     if (tile < q_tiles + k_tiles) {
         const bool is_q = tile < q_tiles;
         const int tt = is_q ? tile : tile - q_tiles;
         const int head = tt / per_head, j0 = (tt % per_head) * 32;
-        *m0 = *m1 = is_q ? a.tm_w[0] : a.tm_w[1];
-        *r0 = head * hd + j0;
-        *r1 = head * hd + half + j0;
-        return;
+        const int sm = is_q ? 0 : 1;
+        return {sm, head * hd + j0, sm, head * hd + half + j0};
     }
-    *m0 = *m1 = a.tm_w[2];
-    *r0 = (tile - q_tiles - k_tiles) * kTileRows;
-    *r1 = *r0 + 32;
+    const int r = (tile - q_tiles - k_tiles) * kTileRows;
+    return {2, r, 2, r + 32};
 }
 
 __device__ __forceinline__ int unit_kboxes(const GemmArgs& a, int u) {
@@ -273,9 +268,10 @@ __device__ __forceinline__ int unit_kboxes(const GemmArgs& a, int u) {
 template <int R>
 __device__ __forceinline__ void tma_weights(const GemmArgs& a, int epi, int u, unsigned char* st, uint64_t* bar) {
     const int tile = u / a.n_chunks, k0 = (u - tile * a.n_chunks) * KC;
-    const void *m0, *m1;
-    int r0, r1;
-    tile_halves(a, epi, tile, &m0, &r0, &m1, &r1);
+    const Halves hv = tile_halves(a, epi, tile);
+    const void* m0 = a.tm_w[hv.s0];
+    const void* m1 = a.tm_w[hv.s1];
+    const int r0 = hv.r0, r1 = hv.r1;
     if (a.wide) {
         mbar_expect_tx(bar, 32768u);
         tma_load_3d(st, m0, 0, k0 >> 6, r0, bar);
@@ -311,8 +307,8 @@ __device__ __forceinline__ void tma_inputs(const GemmArgs& a, int u, unsigned ch
 // parity of the next "empty" completion of stage s to wait for.  Consumers:
 // cphase bit s = parity of the next "full" completion.
 struct Pipe {
-    uint64_t* full;   // [S] TMA completion (count 1: the producer's arrive)
-    uint64_t* empty;  // [S] stage released (count 8: one arrive per consumer warp)
+    uint64_t* full;   // [stages] TMA completion (count 1: the producer's arrive)
+    uint64_t* empty;  // [stages] stage released (count 8: one arrive per consumer warp)
     unsigned pphase;
     unsigned cphase;
 };
@@ -325,7 +321,8 @@ __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, P
     my_units(a.n_units, &u_begin, &n_my);
     if (threadIdx.x == kConsumers) {
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        for (int s = 0; s < S && s < n_my; ++s) {
+        prefetch_tmap(a.tm_x[R == 1 ? 0 : (R == 8 ? 1 : 2)]);
+        for (int s = 0; s < GemmSmem<R>::S && s < n_my; ++s) {
             if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return false;
             pp.pphase ^= 1u << s;
             tma_weights<R>(a, epi, u_begin + s, smem + s * GemmSmem<R>::STAGE, pp.full + s);
@@ -338,12 +335,15 @@ __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, P
 // (one elected thread) streams this CTA's units through the S stages; the 8
 // consumer warps compute and release each stage with one arrival per warp.
 // ut: nullptr, or [64][4] timestamps of this CTA's first units (producer
-// issue, consumer data ready, MMA done, flush done) - a profiling aid.
+// issue, consumer data ready, MMA done, flush done); ct: nullptr, or this
+// CTA's op stamps (FwdParams::trace) - profiling aids.
 template <int R>
 __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefetched, unsigned char* smem,
-                        float* r_s, Pipe& pp, int* err, unsigned long long* ut) {
+                        float* r_s, Pipe& pp, const FwdOp* nx, int* err, unsigned long long* ut,
+                        unsigned long long* ct) {
     using L = GemmSmem<R>;
     constexpr int NT = L::NT, RC = L::RC;
+    constexpr int S = L::S;
     float* red = reinterpret_cast<float*>(smem + S * L::STAGE);  // [64][RC]
     float* ys = red + kTileRows * RC;                             // [64][16]
     __shared__ int s_last;
@@ -353,7 +353,7 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
     int u_begin, n_my;
     my_units(U, &u_begin, &n_my);
 
-    if (threadIdx.x >= kConsumers) {  // producer warp
+    if (threadIdx.x >= kConsumers) {  // producer warp: one elected thread drives the ring
         if (threadIdx.x != kConsumers) return true;
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         for (int i = 0; i < n_my; ++i) {
@@ -370,17 +370,20 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         return true;
     }
 
-    if (threadIdx.x < M) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // 1 / rms of each input row from the previous op's per-tile sums of
+    // squares (fixed order for every M: lane-strided sums, then a shuffle tree)
+    for (int m = warp; m < M; m += kConsumers / 32) {
         float r = 1.f;
         if (a.ss_in) {
             float sum = 0.f;
-            for (int t = 0; t < a.ss_in_tiles; ++t) sum += __ldcg(a.ss_in + threadIdx.x * a.ss_in_tiles + t);
+            for (int t = lane; t < a.ss_in_tiles; t += 32) sum += __ldcg(a.ss_in + m * a.ss_in_tiles + t);
+            sum = warp_sum(sum);
             r = rsqrtf(sum * a.inv_dim + a.eps);
         }
-        r_s[threadIdx.x] = r;
+        if (lane == 0) r_s[m] = r;
     }
 
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int rg = warp & 3, kh = warp >> 2;
     const int g = lane >> 2, tig = lane & 3;
     const int r0 = rg * 16 + g;
@@ -400,7 +403,10 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         const unsigned char* x_s = w_s + L::WB;
         if (!mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err)) return false;
         pp.cphase ^= 1u << s;
-        if (ut && i < 64 && threadIdx.x == 0) ut[i * 4 + 1] = globaltimer();
+        if (threadIdx.x == 0) {
+            if (ut && i < 64) ut[i * 4 + 1] = globaltimer();
+            if (ct && i == 0) ct[1] = globaltimer();
+        }
 
         // A: weight rows r0, r0 + 8; B: input rows nt*8 + g.  Both operands use
         // the same chunk -> logical-k mapping, so the product is unchanged;
@@ -425,7 +431,13 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(pp.empty + s);  // this warp is done with the stage
-        if (ut && i < 64 && threadIdx.x == 0) ut[i * 4 + 2] = globaltimer();
+        if (threadIdx.x == 0) {
+            if (ut && i < 64) ut[i * 4 + 2] = globaltimer();
+            if (ct && i == n_my - 1) {
+                ct[2] = globaltimer();
+                ct[6] = (unsigned long long)n_my;
+            }
+        }
 
         if (!(i == n_my - 1 || chunk == a.n_chunks - 1)) continue;
 
@@ -587,141 +599,178 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 // ---------------------------------------------------------------------------
 // attention op: units (KV head, 64-position chunk)
 // ---------------------------------------------------------------------------
+// Each CTA takes a contiguous run of units.  K / V rows of a unit are copied
+// (cp.async, L2) into one of kAttnBufs ring buffers, so the copies of the next
+// units are in flight while one is computed.  Per unit, for its G * M query
+// vectors v (G query heads of the KV head, M rows): scores (one thread per
+// (v, position)), softmax partial (one warp per v), P V (one thread per (v,
+// dimension pair)); the partial (o, max, sum) goes to global memory.  After
+// its units, a CTA adds its count to each KV head's counter; the last arrival
+// combines the chunk partials of that head in chunk order (flash-decoding
+// style split of the softmax over position chunks).  Every reduction has a
+// fixed order that depends only on the row's own position, not on M.
+constexpr int kAttnBufs = 3;
+
 template <int HD>
 __device__ void attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem) {
     constexpr int KP = HD * 2 + 16;  // bytes per cached row in smem (conflict-free)
-    constexpr int EPL = HD / 32;     // output dims per lane
+    constexpr int EPL = HD / 32;     // output dims per lane in the combine
     constexpr int CPR = HD * 2 / 16;
+    constexpr int BUF = 2 * kAttnChunk * KP;
     const int G = a.n_heads / a.n_kv_heads, NV = G * M;
     const int n_ch = (pos0 + M + kAttnChunk - 1) / kAttnChunk;  // chunks holding any visible position
     const long long U = (long long)a.n_kv_heads * n_ch, GR = gridDim.x;
     const int u_begin = (int)((long long)blockIdx.x * U / GR);
     const int u_end = (int)((long long)(blockIdx.x + 1) * U / GR);
-    unsigned char* ks = smem;
-    unsigned char* vs = ks + kAttnChunk * KP;
-    float* qs = reinterpret_cast<float*>(vs + kAttnChunk * KP);  // [NV][HD]
-    float* sc = qs + NV * HD;                                     // [8][64]
+    float* qs = reinterpret_cast<float*>(smem + kAttnBufs * BUF);  // [NV][HD]
+    float* sc = qs + NV * HD;                                        // [NV][64] scores, then weights
     __shared__ int s_last;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const bool wk = tid < kAttnThreads;  // the producer warp only joins the barriers
+    const size_t part_v = HD + 2;        // floats per partial: o[HD], max, sum
 
-    for (int u = u_begin; u < u_end; ++u) {
-        const int kvh = u / n_ch, c = u - kvh * n_ch;
-        const int t0 = c * kAttnChunk;
-        const int t_end = min(t0 + kAttnChunk, pos0 + M);
-        float* part = a.part + ((size_t)kvh * a.n_chunks) * NV * (HD + 2);
-        const int nt = t_end - t0;
+    auto issue = [&](int u, int b) {
+        const int kvh = u / n_ch, t0 = (u - kvh * n_ch) * kAttnChunk;
+        const int nt = min(t0 + kAttnChunk, pos0 + M) - t0;
         const f16* kb = a.k_cache + ((size_t)kvh * a.max_seq + t0) * HD;
         const f16* vb = a.v_cache + ((size_t)kvh * a.max_seq + t0) * HD;
-        const bool wk = threadIdx.x < kAttnThreads;  // the producer warp only joins the barriers
-        for (int i = wk ? threadIdx.x : nt * CPR; i < nt * CPR; i += kAttnThreads) {
+        unsigned char* ks = smem + b * BUF;
+        unsigned char* vs = ks + kAttnChunk * KP;
+        for (int i = tid; i < nt * CPR; i += kAttnThreads) {
             const int t = i / CPR, cc = i - t * CPR;
             cp_async16(ks + t * KP + cc * 16, kb + (size_t)t * HD + cc * 8, 16);
             cp_async16(vs + t * KP + cc * 16, vb + (size_t)t * HD + cc * 8, 16);
         }
+    };
+    // prologue: one commit group per ring slot (possibly empty), in unit order
+    for (int j = 0; j < kAttnBufs; ++j) {
+        if (wk && u_begin + j < u_end) issue(u_begin + j, j);
         cp_async_commit();
-        for (int i = wk ? threadIdx.x : NV * HD; i < NV * HD; i += kAttnThreads) {
-            const int v = i / HD, e = i - v * HD;
-            const int m = v / G, gi = v - m * G;
-            qs[i] = __ldcg(a.q + (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e);
+    }
+    int q_kvh = -1;
+    for (int u = u_begin; u < u_end; ++u) {
+        const int j = u - u_begin, b = j % kAttnBufs;
+        const int kvh = u / n_ch, c = u - kvh * n_ch, t0 = c * kAttnChunk;
+        const unsigned char* ks = smem + b * BUF;
+        const unsigned char* vs = ks + kAttnChunk * KP;
+        float* part = a.part + (size_t)kvh * a.n_chunks * NV * part_v;
+        if (kvh != q_kvh) {  // q of this KV head's G query heads, M rows (written by other CTAs: L2)
+            for (int i = wk ? tid : NV * HD; i < NV * HD; i += kAttnThreads) {
+                const int v = i / HD, e = i - v * HD;
+                const int m = v / G, gi = v - m * G;
+                qs[i] = __ldcg(a.q + (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e);
+            }
+            q_kvh = kvh;
         }
-        cp_async_wait<0>();
+        cp_async_wait<kAttnBufs - 1>();  // groups retire in order: unit u's copies have landed
         __syncthreads();
 
+        // scores: thread per (v, t); row m sees positions <= pos0 + m
+        for (int i = wk ? tid : NV * kAttnChunk; i < NV * kAttnChunk; i += kAttnThreads) {
+            const int v = i / kAttnChunk, t = i - v * kAttnChunk;
+            const int m = v / G;
+            float dot = -INFINITY;
+            if (t0 + t <= pos0 + m) {
+                dot = 0.f;
+                const unsigned char* kr = ks + t * KP;
+                const float* q = qs + v * HD;
+#pragma unroll
+                for (int e8 = 0; e8 < HD / 8; ++e8) {
+                    const uint4 kv = *reinterpret_cast<const uint4*>(kr + e8 * 16);
+                    const float* qq = q + e8 * 8;
+                    const float2 k0 = f16x2(kv.x), k1 = f16x2(kv.y), k2 = f16x2(kv.z), k3 = f16x2(kv.w);
+                    dot += qq[0] * k0.x + qq[1] * k0.y;
+                    dot += qq[2] * k1.x + qq[3] * k1.y;
+                    dot += qq[4] * k2.x + qq[5] * k2.y;
+                    dot += qq[6] * k3.x + qq[7] * k3.y;
+                }
+                dot *= a.scale;
+            }
+            sc[i] = dot;
+        }
+        __syncthreads();
+
+        // softmax partial: warp per v (positions lane, lane + 32)
         for (int v = wk ? warp : NV; v < NV; v += kAttnThreads / 32) {
             const int m = v / G;
-            const int n_t = min(t_end, pos0 + m + 1) - t0;  // positions this row sees here
-            float* out = part + ((size_t)c * NV + v) * (HD + 2);
-            if (n_t <= 0) {
-                for (int e = lane; e < HD; e += 32) out[e] = 0.f;
+            float* out = part + ((size_t)c * NV + v) * part_v;
+            float* sv = sc + v * kAttnChunk;
+            if (pos0 + m < t0) {  // nothing visible in this chunk
+                sv[lane] = sv[lane + 32] = 0.f;
                 if (lane == 0) { out[HD] = -INFINITY; out[HD + 1] = 0.f; }
                 continue;
             }
-            const float* q = qs + v * HD;
-            float s[2];
-#pragma unroll
-            for (int i = 0; i < 2; ++i) {
-                const int t = lane + 32 * i;
-                float dot = -INFINITY;
-                if (t < n_t) {
-                    dot = 0.f;
-                    const unsigned char* kr = ks + t * KP;
-#pragma unroll
-                    for (int e8 = 0; e8 < HD / 8; ++e8) {
-                        const uint4 kv = *reinterpret_cast<const uint4*>(kr + e8 * 16);
-                        const float* qq = q + e8 * 8;
-                        const float2 k0 = f16x2(kv.x), k1 = f16x2(kv.y), k2 = f16x2(kv.z), k3 = f16x2(kv.w);
-                        dot += qq[0] * k0.x + qq[1] * k0.y;
-                        dot += qq[2] * k1.x + qq[3] * k1.y;
-                        dot += qq[4] * k2.x + qq[5] * k2.y;
-                        dot += qq[6] * k3.x + qq[7] * k3.y;
-                    }
-                    dot *= a.scale;
-                }
-                s[i] = dot;
-            }
-            const float mx = warp_max(fmaxf(s[0], s[1]));
-            const float p0 = lane < n_t ? expf(s[0] - mx) : 0.f;
-            const float p1 = lane + 32 < n_t ? expf(s[1] - mx) : 0.f;
+            const float s0 = sv[lane], s1 = sv[lane + 32];
+            const float mx = warp_max(fmaxf(s0, s1));
+            const float p0 = s0 == -INFINITY ? 0.f : expf(s0 - mx);
+            const float p1 = s1 == -INFINITY ? 0.f : expf(s1 - mx);
             const float l = warp_sum(p0 + p1);
-            float* sw = sc + warp * kAttnChunk;
-            sw[lane] = p0;
-            sw[lane + 32] = p1;
-            __syncwarp();
-            float o[EPL];
-#pragma unroll
-            for (int e = 0; e < EPL; ++e) o[e] = 0.f;
-            for (int t = 0; t < n_t; ++t) {
-                const float w = sw[t];
-                const unsigned char* vr = vs + t * KP + lane * EPL * 2;
-                if constexpr (EPL == 4) {
-                    const uint2 vv = *reinterpret_cast<const uint2*>(vr);
-                    const float2 v0 = f16x2(vv.x), v1 = f16x2(vv.y);
-                    o[0] += w * v0.x;
-                    o[1] += w * v0.y;
-                    o[2] += w * v1.x;
-                    o[3] += w * v1.y;
-                } else {
-                    const float2 v0 = f16x2(*reinterpret_cast<const uint32_t*>(vr));
-                    o[0] += w * v0.x;
-                    o[1] += w * v0.y;
-                }
-            }
-            __syncwarp();
-#pragma unroll
-            for (int e = 0; e < EPL; ++e) out[lane * EPL + e] = o[e];
+            sv[lane] = p0;
+            sv[lane + 32] = p1;
             if (lane == 0) { out[HD] = mx; out[HD + 1] = l; }
         }
-
-        __threadfence();
         __syncthreads();
-        if (threadIdx.x == 0) {
-            const unsigned prev = atomicAdd(&a.counters[kvh], 1u);
-            s_last = prev == (unsigned)(n_ch - 1);
+
+        // P V: thread per (v, dimension pair), positions in order
+        for (int i = wk ? tid : NV * (HD / 2); i < NV * (HD / 2); i += kAttnThreads) {
+            const int v = i / (HD / 2), e2 = i - v * (HD / 2);
+            const int m = v / G;
+            const int n_t = min(kAttnChunk, pos0 + m + 1 - t0);  // <= 0: nothing visible
+            const float* pv = sc + v * kAttnChunk;
+            float o0 = 0.f, o1 = 0.f;
+            for (int t = 0; t < n_t; ++t) {
+                const float w = pv[t];
+                const float2 vv = f16x2(*reinterpret_cast<const uint32_t*>(vs + t * KP + e2 * 4));
+                o0 += w * vv.x;
+                o1 += w * vv.y;
+            }
+            float* out = part + ((size_t)c * NV + v) * part_v;
+            *reinterpret_cast<float2*>(out + 2 * e2) = make_float2(o0, o1);
+        }
+        __syncthreads();  // ring slot b and the score buffer are free
+        if (wk && u + kAttnBufs < u_end) issue(u + kAttnBufs, b);
+        cp_async_commit();
+    }
+    if (u_begin >= u_end) return;
+
+    // publish the partials; per KV head, the CTA that completes the count combines
+    __threadfence();
+    __syncthreads();
+    for (int kvh = u_begin / n_ch; kvh <= (u_end - 1) / n_ch; ++kvh) {
+        const int cnt = min(u_end, (kvh + 1) * n_ch) - max(u_begin, kvh * n_ch);
+        if (tid == 0) {
+            const unsigned prev = atomicAdd(&a.counters[kvh], (unsigned)cnt);
+            s_last = prev + (unsigned)cnt == (unsigned)n_ch;
         }
         __syncthreads();
         if (s_last) {
             __threadfence();
-            // combine: row m uses chunks 0 .. (pos0 + m) / 64, in chunk order
+            const float* part = a.part + (size_t)kvh * a.n_chunks * NV * part_v;
+            // row m uses chunks 0 .. (pos0 + m) / 64
             for (int v = wk ? warp : NV; v < NV; v += kAttnThreads / 32) {
                 const int m = v / G, gi = v - m * G;
                 const int nch = (pos0 + m) / kAttnChunk + 1;
                 float mx = -INFINITY;
-                for (int cc = 0; cc < nch; ++cc)
-                    mx = fmaxf(mx, __ldcg(part + ((size_t)cc * NV + v) * (HD + 2) + HD));
-                float L = 0.f;
+                for (int cc = lane; cc < nch; cc += 32) mx = fmaxf(mx, __ldcg(part + ((size_t)cc * NV + v) * part_v + HD));
+                mx = warp_max(mx);
+                float lp = 0.f;
+                for (int cc = lane; cc < nch; cc += 32) {
+                    const float* pp = part + ((size_t)cc * NV + v) * part_v;
+                    const float mc = __ldcg(pp + HD);
+                    if (mc != -INFINITY) lp += expf(mc - mx) * __ldcg(pp + HD + 1);
+                }
+                const float inv = 1.f / warp_sum(lp);
                 float o[EPL];
 #pragma unroll
                 for (int e = 0; e < EPL; ++e) o[e] = 0.f;
+#pragma unroll 4
                 for (int cc = 0; cc < nch; ++cc) {
-                    const float* pp = part + ((size_t)cc * NV + v) * (HD + 2);
+                    const float* pp = part + ((size_t)cc * NV + v) * part_v;
                     const float mc = __ldcg(pp + HD);
-                    if (mc == -INFINITY) continue;
-                    const float f = expf(mc - mx);
-                    L += f * __ldcg(pp + HD + 1);
+                    const float f = mc == -INFINITY ? 0.f : expf(mc - mx);  // empty chunks hold o = 0
 #pragma unroll
                     for (int e = 0; e < EPL; ++e) o[e] += f * __ldcg(pp + lane * EPL + e);
                 }
-                const float inv = 1.f / L;
                 const size_t at = (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + lane * EPL;
 #pragma unroll
                 for (int e = 0; e < EPL; ++e) {
@@ -731,9 +780,9 @@ __device__ void attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem)
                     a.out_lo[at + e] = __float2bfloat16_rn(val - __bfloat162float(vh));
                 }
             }
-            if (threadIdx.x == 0) a.counters[kvh] = 0u;
+            if (tid == 0) a.counters[kvh] = 0u;
         }
-        __syncthreads();  // smem reused by the next unit
+        __syncthreads();
     }
 }
 
@@ -795,6 +844,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     __shared__ float r_s[kMaxRows];
     __shared__ int s_pos0, s_fail;
+    constexpr int S = GemmSmem<R>::S;
     __shared__ __align__(8) uint64_t full[S];   // TMA completion per stage
     __shared__ __align__(8) uint64_t empty[S];  // stage released by the 8 consumer warps
     __shared__ FwdOp s_op[2];                   // current and next op's arguments
@@ -828,19 +878,26 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         const FwdOp& op = s_op[o & 1];
         const int type = op.type;
         bool ok = true;
-        if (type == OP_EMBED) embed_op(p, pos0);
-        else if (type == OP_ATTN) attn_op<HD>(op.at, p.M, pos0, smem);
-        else
-            ok = gemm_op<R>(op.g, epi_of(type), p.M, pos0, prefetched, smem, r_s, pp, p.err,
-                            (p.trace && blockIdx.x == 0 && o == 1) ? p.trace + 1024 : nullptr);
-        prefetched = false;
+        unsigned long long* ct = (p.trace && o == p.trace_op) ? p.trace + kTraceCtas + blockIdx.x * 8 : nullptr;
+        if (ct && threadIdx.x == 0) ct[0] = globaltimer();
+        // the next op's arguments (its slot held op o-1, finished by every thread)
+        const FwdOp* nx = nullptr;
         if (o + 1 < p.n_ops) {
             copy_op(p.ops + o + 1, s_op + ((o + 1) & 1));  // (all threads, includes a barrier)
-            const FwdOp& nx = s_op[(o + 1) & 1];
-            if (ok && is_gemm(nx.type)) {
-                ok = gemm_prefetch<R>(nx.g, epi_of(nx.type), smem, pp, p.err);
-                prefetched = true;
-            }
+            nx = s_op + ((o + 1) & 1);
+        }
+        if (is_gemm(type)) {
+            ok = gemm_op<R>(op.g, epi_of(type), p.M, pos0, prefetched, smem, r_s, pp, nx, p.err,
+                            (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr, ct);
+        } else {
+            if (type == OP_EMBED) embed_op(p, pos0);
+            else attn_op<HD>(op.at, p.M, pos0, smem);
+        }
+        if (ct && threadIdx.x == 0) ct[3] = globaltimer();
+        prefetched = false;
+        if (nx && ok && is_gemm(nx->type)) {
+            ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err);
+            prefetched = true;
         }
         if (!ok) s_fail = 1;
         __syncthreads();
@@ -848,6 +905,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
             drain_before_exit();
             return;
         }
+        if (ct && threadIdx.x == 0) ct[4] = globaltimer();
         if (o + 1 < p.n_ops) {
             target += gridDim.x;
             if (!grid_barrier(p.bar, target, p.err)) {
@@ -855,6 +913,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
                 return;
             }
         }
+        if (ct && threadIdx.x == 0) ct[5] = globaltimer();
         if (p.trace && blockIdx.x == 0 && threadIdx.x == 0) p.trace[o + 1] = globaltimer();
     }
 }
@@ -888,7 +947,7 @@ size_t forward_smem_bytes(int M) {
 }
 
 size_t attention_smem_bytes(int head_dim, int group, int M) {
-    return 2 * kAttnChunk * (head_dim * 2 + 16) + (size_t)group * M * head_dim * 4 + 8 * kAttnChunk * 4;
+    return (size_t)kAttnBufs * 2 * kAttnChunk * (head_dim * 2 + 16) + (size_t)group * M * (head_dim + kAttnChunk) * 4;
 }
 
 int forward_configure() {

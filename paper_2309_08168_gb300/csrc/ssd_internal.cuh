@@ -18,7 +18,7 @@ constexpr int kGemmThreads = 256; // 8 warps: 4 row groups x 2 k-interleaves
 constexpr int kAttnChunk = 64;    // KV positions per attention CTA (absolute chunks)
 constexpr int kAttnThreads = 256;
 constexpr int kStreamKC = 256;    // k per streaming-GEMM work unit (64 rows x 256 = 32 KB of weights)
-constexpr int kStreamStages = 4;  // cp.async ring depth of the streaming GEMM
+constexpr int kTraceUnits = 1024, kTraceCtas = 1280;  // offsets in FwdParams::trace
 
 // ---------------------------------------------------------------------------
 // device state of the decode loop (one per handle, in device memory)
@@ -141,7 +141,13 @@ struct FwdParams {
     float* ss;            // per-64-column sums of h^2 [16][d/64]
     unsigned* bar;        // grid-barrier counter, zero at launch
     int* err;             // device error code
-    unsigned long long* trace;  // nullptr, or [n_ops + 1] globaltimer stamps (start, end of op o)
+    // Profiling hook: nullptr, or globaltimer stamps: [0, n_ops] start, end of
+    // op o (CTA 0); [1024, 1280) CTA 0's first 64 units of op trace_op (producer
+    // issue, data ready, MMA done, flush done); [1280, 1280 + 8 * grid) per CTA,
+    // op trace_op: start, first data ready, last MMA done, work done, barrier
+    // arrive, barrier release, number of units, 0.
+    unsigned long long* trace;
+    int trace_op;
 };
 
 int forward_configure();
