@@ -317,18 +317,21 @@ struct Pipe {
 // before the grid barrier (they do not depend on the previous op).
 template <int R>
 __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, Pipe& pp, int* err) {
+    constexpr int S = GemmSmem<R>::S;
     int u_begin, n_my;
     my_units(a.n_units, &u_begin, &n_my);
+    bool ok = true;
     if (threadIdx.x == kConsumers) {
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         prefetch_tmap(a.tm_x[R == 1 ? 0 : (R == 8 ? 1 : 2)]);
-        for (int s = 0; s < GemmSmem<R>::S && s < n_my; ++s) {
-            if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return false;
+        for (int s = 0; s < S && s < n_my && ok; ++s) {
+            ok = mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err);
+            if (!ok) break;
             pp.pphase ^= 1u << s;
             tma_weights<R>(a, epi, u_begin + s, smem + s * GemmSmem<R>::STAGE, pp.full + s);
         }
     }
-    return true;
+    return ok;
 }
 
 // Returns false if a TMA wait timed out (error recorded).  The producer warp
@@ -480,6 +483,19 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         }
         consumer_sync();
 
+        // RESID: this tile's residual h (written by earlier ops: L2), loaded
+        // before the split-K exchange so its latency overlaps it
+        constexpr int HJ = kMaxRows * kTileRows / kGemmThreads;
+        float hpre[HJ];
+        if (epi == EPI_RESID) {
+#pragma unroll
+            for (int j = 0; j < HJ; ++j) {
+                const int idx = threadIdx.x + j * kGemmThreads;
+                const int m = idx / kTileRows, n = tile * kTileRows + (idx - m * kTileRows);
+                hpre[j] = (idx < M * kTileRows && n < a.N) ? __ldcg(a.out_f32 + (size_t)m * a.ldo + n) : 0.f;
+            }
+        }
+
         // segments of other CTAs: the last one to arrive sums all in order
         const long long u_first = (long long)tile * a.n_chunks;
         const int seg0 = unit_owner(u_first, U, G);
@@ -504,6 +520,7 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
                 const int m = idx / kTileRows, r = idx - m * kTileRows;
                 const float* p = slots + m * kTileRows + r;
                 float sum = __ldcg(p);
+#pragma unroll 4
                 for (int sg = 1; sg < nseg; ++sg) sum += __ldcg(p + (size_t)sg * kMaxRows * kTileRows);
                 ys[r * 16 + m] = sum;
             }
@@ -519,13 +536,16 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
                 if (n < a.N) a.out_f32[(size_t)m * a.ldo + n] = ys[r * 16 + m] * r_s[m];
             }
         } else if (epi == EPI_RESID) {
-            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+#pragma unroll
+            for (int j = 0; j < HJ; ++j) {
+                const int idx = threadIdx.x + j * kGemmThreads;
+                if (idx >= M * kTileRows) break;
                 const int m = idx / kTileRows, r = idx - m * kTileRows;
                 const int n = tile * kTileRows + r;
                 float hv = 0.f;
                 if (n < a.N) {
                     float* o = a.out_f32 + (size_t)m * a.ldo + n;
-                    hv = __ldcg(o) + ys[r * 16 + m];  // L2: other CTAs wrote h in earlier ops
+                    hv = hpre[j] + ys[r * 16 + m];
                     *o = hv;
                     if (a.g_next) {
                         const float z = hv * __bfloat162float(a.g_next[n]);
