@@ -183,18 +183,20 @@ size_t trace_words(const ssd_handle* h) { return (size_t)kTraceCtas + 8 * (size_
 
 int tmap_weight(int l, int which) { return 7 * l + which; }
 int tmap_x(const ssd_handle* h, int buf, int cls) { return 7 * h->cfg.n_layers + 1 + buf * 3 + cls; }
+int tmap_kv(const ssd_handle* h, int v) { return 7 * h->cfg.n_layers + 10 + v; }
 
-// Checks the TMA rules and encodes a bf16 tensor map with 64-element (128-byte)
+// Checks the TMA rules and encodes a 16-bit tensor map with 64-element (128-byte)
 // inner boxes, 128-byte swizzle, zero fill out of range: base 16-byte aligned,
 // strides multiples of 16 bytes.
 int encode_map(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* base, int rank,
-               const cuuint64_t* dims, const cuuint64_t* strides, const cuuint32_t* box) {
+               const cuuint64_t* dims, const cuuint64_t* strides, const cuuint32_t* box,
+               CUtensorMapDataType dtype = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
     if ((uintptr_t)base & 15u) return fail(SSD_ERR_INVALID_ARG, "tensor base not 16-byte aligned for TMA");
     for (int i = 0; i + 1 < rank; ++i)
         if (strides[i] % 16) return fail(SSD_ERR_INVALID_ARG, "tensor stride not a multiple of 16 bytes for TMA");
     if (dims[0] < 64 || box[0] != 64) return fail(SSD_ERR_INVALID_ARG, "tensor row shorter than one TMA box");
     cuuint32_t estr[4] = {1, 1, 1, 1};
-    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base), dims, strides,
+    CUresult r = enc(m, dtype, (cuuint32_t)rank, const_cast<void*>(base), dims, strides,
                      box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return fail(SSD_ERR_CUDA, "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")");
@@ -257,6 +259,14 @@ int build_tmaps(ssd_handle* h) {
     for (int b = 0; b < 3 && !rc; ++b)
         for (int cls = 0; cls < 3 && !rc; ++cls)
             rc = encode_planes(enc, &maps[tmap_x(h, b, cls)], planes[b], widths[b], rows[cls]);
+    // K / V cache [L][Hkv][max_seq][hd] fp16 as {hd, max_seq, L * Hkv}, box 64 dims x 64 positions
+    for (int v = 0; v < 2 && !rc; ++v) {
+        cuuint64_t dims[3] = {(cuuint64_t)c.head_dim, (cuuint64_t)c.max_seq, (cuuint64_t)L * c.n_kv_heads};
+        cuuint64_t strides[2] = {(cuuint64_t)c.head_dim * 2, (cuuint64_t)c.max_seq * c.head_dim * 2};
+        cuuint32_t box[3] = {64, (cuuint32_t)kAttnChunk, 1};
+        rc = encode_map(enc, &maps[tmap_kv(h, v)], v ? h->vc : h->kc, 3, dims, strides, box,
+                        CU_TENSOR_MAP_DATA_TYPE_FLOAT16);
+    }
     if (rc) return rc;
     CUDA_TRY(cudaMemcpy(h->tmaps, maps.data(), maps.size() * sizeof(CUtensorMap), cudaMemcpyHostToDevice),
              "tensor map upload");
@@ -323,7 +333,8 @@ std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
             FwdOp at{};
             at.type = OP_ATTN;
             AttnArgs& t = at.at;
-            t.q = h->q; t.k_cache = a.k_cache; t.v_cache = a.v_cache;
+            t.q = h->q;
+            t.tm_k = h->tmaps + tmap_kv(h, 0); t.tm_v = h->tmaps + tmap_kv(h, 1); t.kv_z0 = l * c.n_kv_heads;
             t.out_hi = h->at_hi; t.out_lo = h->at_lo;
             t.part = h->attn_part; t.counters = h->counters + h->gemm_counters;
             t.n_heads = c.n_heads; t.n_kv_heads = c.n_kv_heads; t.head_dim = c.head_dim;
@@ -512,11 +523,6 @@ int check_config(const ssd_config* c) {
     if (c->max_seq < 2 || c->max_seq > (1 << 24)) return fail(SSD_ERR_INVALID_ARG, "max_seq out of range");
     if (!(c->rms_eps > 0.f) || !(c->rope_theta > 0.f))
         return fail(SSD_ERR_INVALID_ARG, "rms_eps and rope_theta must be positive");
-    const int G = c->n_heads / c->n_kv_heads;
-    if (attention_smem_bytes(c->head_dim, G, 1) > forward_smem_bytes(1) ||
-        attention_smem_bytes(c->head_dim, G, 8) > forward_smem_bytes(8) ||
-        attention_smem_bytes(c->head_dim, G, kMaxRows) > forward_smem_bytes(kMaxRows))
-        return fail(SSD_ERR_INVALID_ARG, "n_heads / n_kv_heads too large");
     return SSD_OK;
 }
 
@@ -656,7 +662,7 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
         return bail(rc);
     h->max_ops = 2 + 5 * L;
     if (h->max_ops + 1 > 1024) return bail(fail(SSD_ERR_INVALID_ARG, "too many layers (at most 204)"));
-    h->n_tmaps = 7 * L + 1 + 9;
+    h->n_tmaps = 7 * L + 1 + 9 + 2;
     if ((rc = dalloc(h, &h->tmaps, (size_t)h->n_tmaps, &B)) ||
         (rc = dalloc(h, &h->ops_full, (size_t)h->max_ops, &B)) ||
         (rc = dalloc(h, &h->ops_draft, (size_t)h->max_ops, &B)) ||

@@ -201,6 +201,11 @@ __device__ __forceinline__ void prefetch_tmap(const void* tmap) {
 // narrow layout (K % 64 != 0, one copy per 64-wide k-box):
 //   weights: [k-box 4][row 64][64]: kbox * 8 KB + r * 128
 //   inputs : [k-box 4][max(2R, 8) rows][64]: kbox * XKB + p * 128
+// Attention unit in a stage: K rows of the 64-position chunk at 0 (dims 0-63,
+// then 64-127 at 8 KB), V rows at 16 KB; position t, 16-byte chunk c of a
+// 64-dim box at box + t * 128 + ((c ^ (t & 7)) << 4).
+// After the ring: the consumers' scratch - split-K reduction buffers of a
+// projection, or (same bytes: one op at a time) q / scores of attention.
 template <int R>
 struct GemmSmem {
     static constexpr int NT = (2 * R + 7) / 8;   // n8 MMA tiles: 1 | 2 | 4
@@ -211,7 +216,14 @@ struct GemmSmem {
     static constexpr int STAGE = WB + XB;
     static constexpr int RC = NT * 8;
     static constexpr int S = 4;  // ring depth (5 or 6 stages, where they fit, measured no faster)
-    static constexpr size_t BYTES = 1024 + (size_t)S * STAGE + kTileRows * RC * 4 + kTileRows * 16 * 4;
+    static constexpr int VG = 16;  // attention: query vectors per pass over a staged chunk
+    static constexpr int RED = S * STAGE;                // [64][RC] floats
+    static constexpr int YS = RED + kTileRows * RC * 4;  // [64][16] floats
+    static constexpr int ATT = RED;                      // [VG][128] q, [VG][64] scores
+    static constexpr int SCRATCH_GEMM = kTileRows * RC * 4 + kTileRows * 16 * 4;
+    static constexpr int SCRATCH_ATT = VG * 128 * 4 + VG * kAttnChunk * 4;
+    static constexpr size_t BYTES =
+        1024 + (size_t)RED + (SCRATCH_GEMM > SCRATCH_ATT ? SCRATCH_GEMM : SCRATCH_ATT);
 };
 
 // byte offset of 16-byte chunk c (0..7) of k-box kb in row r of the weights,
@@ -347,8 +359,8 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
     using L = GemmSmem<R>;
     constexpr int NT = L::NT, RC = L::RC;
     constexpr int S = L::S;
-    float* red = reinterpret_cast<float*>(smem + S * L::STAGE);  // [64][RC]
-    float* ys = red + kTileRows * RC;                             // [64][16]
+    float* red = reinterpret_cast<float*>(smem + L::RED);  // [64][RC]
+    float* ys = reinterpret_cast<float*>(smem + L::YS);    // [64][16]
     __shared__ int s_last;
 
     const long long U = a.n_units, G = op_ctas(U);
@@ -617,167 +629,204 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 }
 
 // ---------------------------------------------------------------------------
-// attention op: units (KV head, 64-position chunk)
+// attention op: units (KV head, 64-position chunk), through the TMA ring
 // ---------------------------------------------------------------------------
-// Each CTA takes a contiguous run of units.  K / V rows of a unit are copied
-// (cp.async, L2) into one of kAttnBufs ring buffers, so the copies of the next
-// units are in flight while one is computed.  Per unit, for its G * M query
-// vectors v (G query heads of the KV head, M rows): scores (one thread per
-// (v, position)), softmax partial (one warp per v), P V (one thread per (v,
-// dimension pair)); the partial (o, max, sum) goes to global memory.  After
-// its units, a CTA adds its count to each KV head's counter; the last arrival
-// combines the chunk partials of that head in chunk order (flash-decoding
-// style split of the softmax over position chunks).  Every reduction has a
-// fixed order that depends only on the row's own position, not on M.
-constexpr int kAttnBufs = 3;
+// Each CTA takes a contiguous run of units.  The producer thread requests the
+// K / V rows of each unit (TMA, 128-byte swizzle) into the ring's stages, so
+// the copies of the next units are in flight while one is computed, and after
+// its last unit it goes on to the next projection's weights.  Per unit, for
+// its G * M query vectors v (G query heads of the KV head, M rows), in passes
+// of up to VG vectors: scores (one thread per (v, position)), softmax
+// partial (one warp per v), P V (one thread per (v, dimension pair)); the
+// partial (o, max, sum) goes to global memory.  After its units, a CTA adds
+// its count to each KV head's counter; the last arrival combines the chunk
+// partials of that head in chunk order (flash-decoding style split of the
+// softmax over position chunks).  Every reduction has a fixed order that
+// depends only on the row's own position, not on M.
+struct AttnRange {
+    int n_ch, u_begin, u_end;
+};
+__device__ __forceinline__ AttnRange attn_range(const AttnArgs& a, int M, int pos0) {
+    AttnRange r;
+    r.n_ch = (pos0 + M + kAttnChunk - 1) / kAttnChunk;  // chunks holding any visible position
+    const long long U = (long long)a.n_kv_heads * r.n_ch, GR = gridDim.x;
+    r.u_begin = (int)((long long)blockIdx.x * U / GR);
+    r.u_end = (int)((long long)(blockIdx.x + 1) * U / GR);
+    return r;
+}
 
-template <int HD>
-__device__ void attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem) {
-    constexpr int KP = HD * 2 + 16;  // bytes per cached row in smem (conflict-free)
-    constexpr int EPL = HD / 32;     // output dims per lane in the combine
-    constexpr int CPR = HD * 2 / 16;
-    constexpr int BUF = 2 * kAttnChunk * KP;
+// Returns false if a wait timed out (error recorded).
+template <int R, int HD>
+__device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem, Pipe& pp, int* err) {
+    using L = GemmSmem<R>;
+    constexpr int S = L::S, VG = L::VG;
+    constexpr int EPL = HD / 32;  // output dims per lane in the combine
     const int G = a.n_heads / a.n_kv_heads, NV = G * M;
-    const int n_ch = (pos0 + M + kAttnChunk - 1) / kAttnChunk;  // chunks holding any visible position
-    const long long U = (long long)a.n_kv_heads * n_ch, GR = gridDim.x;
-    const int u_begin = (int)((long long)blockIdx.x * U / GR);
-    const int u_end = (int)((long long)(blockIdx.x + 1) * U / GR);
-    float* qs = reinterpret_cast<float*>(smem + kAttnBufs * BUF);  // [NV][HD]
-    float* sc = qs + NV * HD;                                        // [NV][64] scores, then weights
+    const AttnRange ar = attn_range(a, M, pos0);
+
+    if (threadIdx.x >= kConsumers) {  // producer warp: one elected thread requests K / V
+        if (threadIdx.x != kConsumers) return true;
+        if (ar.u_begin < ar.u_end) {
+            // K / V rows of this forward were stored by other CTAs (generic proxy)
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+            prefetch_tmap(a.tm_k);
+            prefetch_tmap(a.tm_v);
+        }
+        for (int u = ar.u_begin; u < ar.u_end; ++u) {
+            const int i = u - ar.u_begin, s = i % S;
+            unsigned char* st = smem + s * L::STAGE;
+            const int kvh = u / ar.n_ch, t0 = (u - kvh * ar.n_ch) * kAttnChunk;
+            if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return false;
+            pp.pphase ^= 1u << s;
+            mbar_arrive_expect_tx(pp.full + s, 2u * (HD / 64) * 8192u);
+#pragma unroll
+            for (int bx = 0; bx < HD / 64; ++bx) {
+                tma_load_3d(st + bx * 8192, a.tm_k, bx * 64, t0, a.kv_z0 + kvh, pp.full + s);
+                tma_load_3d(st + 16384 + bx * 8192, a.tm_v, bx * 64, t0, a.kv_z0 + kvh, pp.full + s);
+            }
+        }
+        return true;
+    }
+
+    float* qs = reinterpret_cast<float*>(smem + L::ATT);  // [VG][HD]
+    float* sc = qs + VG * HD;                              // [VG][64] scores, then weights
     __shared__ int s_last;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const bool wk = tid < kAttnThreads;  // the producer warp only joins the barriers
-    const size_t part_v = HD + 2;        // floats per partial: o[HD], max, sum
-
-    auto issue = [&](int u, int b) {
-        const int kvh = u / n_ch, t0 = (u - kvh * n_ch) * kAttnChunk;
-        const int nt = min(t0 + kAttnChunk, pos0 + M) - t0;
-        const f16* kb = a.k_cache + ((size_t)kvh * a.max_seq + t0) * HD;
-        const f16* vb = a.v_cache + ((size_t)kvh * a.max_seq + t0) * HD;
-        unsigned char* ks = smem + b * BUF;
-        unsigned char* vs = ks + kAttnChunk * KP;
-        for (int i = tid; i < nt * CPR; i += kAttnThreads) {
-            const int t = i / CPR, cc = i - t * CPR;
-            cp_async16(ks + t * KP + cc * 16, kb + (size_t)t * HD + cc * 8, 16);
-            cp_async16(vs + t * KP + cc * 16, vb + (size_t)t * HD + cc * 8, 16);
-        }
-    };
-    // prologue: one commit group per ring slot (possibly empty), in unit order
-    for (int j = 0; j < kAttnBufs; ++j) {
-        if (wk && u_begin + j < u_end) issue(u_begin + j, j);
-        cp_async_commit();
-    }
+    const size_t part_v = HD + 2;  // floats per partial: o[HD], max, sum
     int q_kvh = -1;
-    for (int u = u_begin; u < u_end; ++u) {
-        const int j = u - u_begin, b = j % kAttnBufs;
-        const int kvh = u / n_ch, c = u - kvh * n_ch, t0 = c * kAttnChunk;
-        const unsigned char* ks = smem + b * BUF;
-        const unsigned char* vs = ks + kAttnChunk * KP;
+    bool ok = true;
+
+    for (int u = ar.u_begin; u < ar.u_end; ++u) {
+        const int i = u - ar.u_begin, s = i % S;
+        const unsigned char* ks = smem + s * L::STAGE;
+        const unsigned char* vs = ks + 16384;
+        const int kvh = u / ar.n_ch, c = u - kvh * ar.n_ch, t0 = c * kAttnChunk;
         float* part = a.part + (size_t)kvh * a.n_chunks * NV * part_v;
-        if (kvh != q_kvh) {  // q of this KV head's G query heads, M rows (written by other CTAs: L2)
-            for (int i = wk ? tid : NV * HD; i < NV * HD; i += kAttnThreads) {
-                const int v = i / HD, e = i - v * HD;
-                const int m = v / G, gi = v - m * G;
-                qs[i] = __ldcg(a.q + (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e);
-            }
-            q_kvh = kvh;
-        }
-        cp_async_wait<kAttnBufs - 1>();  // groups retire in order: unit u's copies have landed
-        __syncthreads();
-
-        // scores: thread per (v, t); row m sees positions <= pos0 + m
-        for (int i = wk ? tid : NV * kAttnChunk; i < NV * kAttnChunk; i += kAttnThreads) {
-            const int v = i / kAttnChunk, t = i - v * kAttnChunk;
-            const int m = v / G;
-            float dot = -INFINITY;
-            if (t0 + t <= pos0 + m) {
-                dot = 0.f;
-                const unsigned char* kr = ks + t * KP;
-                const float* q = qs + v * HD;
-#pragma unroll
-                for (int e8 = 0; e8 < HD / 8; ++e8) {
-                    const uint4 kv = *reinterpret_cast<const uint4*>(kr + e8 * 16);
-                    const float* qq = q + e8 * 8;
-                    const float2 k0 = f16x2(kv.x), k1 = f16x2(kv.y), k2 = f16x2(kv.z), k3 = f16x2(kv.w);
-                    dot += qq[0] * k0.x + qq[1] * k0.y;
-                    dot += qq[2] * k1.x + qq[3] * k1.y;
-                    dot += qq[4] * k2.x + qq[5] * k2.y;
-                    dot += qq[6] * k3.x + qq[7] * k3.y;
+        ok = mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err) && ok;
+        pp.cphase ^= 1u << s;
+        for (int v0 = 0; v0 < NV; v0 += VG) {
+            const int nv = min(VG, NV - v0);
+            if (kvh != q_kvh || NV > VG) {  // q of this pass (written by other CTAs: L2)
+                for (int k = tid; k < nv * HD; k += kConsumers) {
+                    const int v = v0 + k / HD, e = k % HD;
+                    const int m = v / G, gi = v - m * G;
+                    qs[k] = __ldcg(a.q + (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e);
                 }
-                dot *= a.scale;
+                q_kvh = kvh;
+                consumer_sync();
             }
-            sc[i] = dot;
-        }
-        __syncthreads();
+            // scores: thread per (v, t); row m sees positions <= pos0 + m
+            for (int k = tid; k < nv * kAttnChunk; k += kConsumers) {
+                const int vl = k / kAttnChunk, t = k - vl * kAttnChunk;
+                const int m = (v0 + vl) / G;
+                float dot = -INFINITY;
+                if (t0 + t <= pos0 + m) {
+                    float d0 = 0.f, d1 = 0.f;
+                    const float* q = qs + vl * HD;
+                    const int sw = t & 7;
+#pragma unroll
+                    for (int bx = 0; bx < HD / 64; ++bx) {
+#pragma unroll
+                        for (int cc = 0; cc < 8; ++cc) {
+                            const uint4 kv =
+                                *reinterpret_cast<const uint4*>(ks + bx * 8192 + t * 128 + ((cc ^ sw) << 4));
+                            const float* qq = q + bx * 64 + cc * 8;
+                            const float2 k0 = f16x2(kv.x), k1 = f16x2(kv.y), k2 = f16x2(kv.z), k3 = f16x2(kv.w);
+                            float& d = (cc & 1) ? d1 : d0;
+                            d += qq[0] * k0.x + qq[1] * k0.y;
+                            d += qq[2] * k1.x + qq[3] * k1.y;
+                            d += qq[4] * k2.x + qq[5] * k2.y;
+                            d += qq[6] * k3.x + qq[7] * k3.y;
+                        }
+                    }
+                    dot = (d0 + d1) * a.scale;
+                }
+                sc[k] = dot;
+            }
+            consumer_sync();
 
-        // softmax partial: warp per v (positions lane, lane + 32)
-        for (int v = wk ? warp : NV; v < NV; v += kAttnThreads / 32) {
-            const int m = v / G;
-            float* out = part + ((size_t)c * NV + v) * part_v;
-            float* sv = sc + v * kAttnChunk;
-            if (pos0 + m < t0) {  // nothing visible in this chunk
-                sv[lane] = sv[lane + 32] = 0.f;
-                if (lane == 0) { out[HD] = -INFINITY; out[HD + 1] = 0.f; }
-                continue;
+            // softmax partial: warp per v (positions lane, lane + 32)
+            for (int vl = warp; vl < nv; vl += kConsumers / 32) {
+                const int v = v0 + vl, m = v / G;
+                float* o = part + ((size_t)c * NV + v) * part_v;
+                float* sv = sc + vl * kAttnChunk;
+                if (pos0 + m < t0) {  // nothing visible in this chunk
+                    sv[lane] = sv[lane + 32] = 0.f;
+                    if (lane == 0) { o[HD] = -INFINITY; o[HD + 1] = 0.f; }
+                    continue;
+                }
+                const float s0 = sv[lane], s1 = sv[lane + 32];
+                const float mx = warp_max(fmaxf(s0, s1));
+                const float p0 = s0 == -INFINITY ? 0.f : expf(s0 - mx);
+                const float p1 = s1 == -INFINITY ? 0.f : expf(s1 - mx);
+                const float l = warp_sum(p0 + p1);
+                sv[lane] = p0;
+                sv[lane + 32] = p1;
+                if (lane == 0) { o[HD] = mx; o[HD + 1] = l; }
             }
-            const float s0 = sv[lane], s1 = sv[lane + 32];
-            const float mx = warp_max(fmaxf(s0, s1));
-            const float p0 = s0 == -INFINITY ? 0.f : expf(s0 - mx);
-            const float p1 = s1 == -INFINITY ? 0.f : expf(s1 - mx);
-            const float l = warp_sum(p0 + p1);
-            sv[lane] = p0;
-            sv[lane + 32] = p1;
-            if (lane == 0) { out[HD] = mx; out[HD + 1] = l; }
-        }
-        __syncthreads();
+            consumer_sync();
 
-        // P V: thread per (v, dimension pair), positions in order
-        for (int i = wk ? tid : NV * (HD / 2); i < NV * (HD / 2); i += kAttnThreads) {
-            const int v = i / (HD / 2), e2 = i - v * (HD / 2);
-            const int m = v / G;
-            const int n_t = min(kAttnChunk, pos0 + m + 1 - t0);  // <= 0: nothing visible
-            const float* pv = sc + v * kAttnChunk;
-            float o0 = 0.f, o1 = 0.f;
-            for (int t = 0; t < n_t; ++t) {
-                const float w = pv[t];
-                const float2 vv = f16x2(*reinterpret_cast<const uint32_t*>(vs + t * KP + e2 * 4));
-                o0 += w * vv.x;
-                o1 += w * vv.y;
+            // P V: thread per (v, dimension pair), even and odd positions in
+            // two accumulator pairs, summed at the end
+            for (int k = tid; k < nv * (HD / 2); k += kConsumers) {
+                const int vl = k / (HD / 2), e2 = k - vl * (HD / 2);
+                const int v = v0 + vl, m = v / G;
+                const int n_t = min(kAttnChunk, pos0 + m + 1 - t0);  // <= 0: nothing visible
+                const float* pv = sc + vl * kAttnChunk;
+                const int e = 2 * e2, bx = e >> 6, cc = (e & 63) >> 3, off = (e & 7) * 2;
+                const unsigned char* vb = vs + bx * 8192 + off;
+                float a0 = 0.f, a1 = 0.f, b0 = 0.f, b1 = 0.f;
+                int t = 0;
+                for (; t + 1 < n_t; t += 2) {
+                    const float2 va = f16x2(*reinterpret_cast<const uint32_t*>(vb + t * 128 + ((cc ^ (t & 7)) << 4)));
+                    const float2 vn =
+                        f16x2(*reinterpret_cast<const uint32_t*>(vb + (t + 1) * 128 + ((cc ^ ((t + 1) & 7)) << 4)));
+                    a0 += pv[t] * va.x;
+                    a1 += pv[t] * va.y;
+                    b0 += pv[t + 1] * vn.x;
+                    b1 += pv[t + 1] * vn.y;
+                }
+                if (t < n_t) {
+                    const float2 va = f16x2(*reinterpret_cast<const uint32_t*>(vb + t * 128 + ((cc ^ (t & 7)) << 4)));
+                    a0 += pv[t] * va.x;
+                    a1 += pv[t] * va.y;
+                }
+                float* o = part + ((size_t)c * NV + v) * part_v;
+                *reinterpret_cast<float2*>(o + e) = make_float2(a0 + b0, a1 + b1);
             }
-            float* out = part + ((size_t)c * NV + v) * part_v;
-            *reinterpret_cast<float2*>(out + 2 * e2) = make_float2(o0, o1);
+            consumer_sync();  // scores / q of this pass are free
         }
-        __syncthreads();  // ring slot b and the score buffer are free
-        if (wk && u + kAttnBufs < u_end) issue(u + kAttnBufs, b);
-        cp_async_commit();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(pp.empty + s);  // the stage is free
     }
-    if (u_begin >= u_end) return;
+    if (ar.u_begin >= ar.u_end) return ok;
 
     // publish the partials; per KV head, the CTA that completes the count combines
     __threadfence();
-    __syncthreads();
-    for (int kvh = u_begin / n_ch; kvh <= (u_end - 1) / n_ch; ++kvh) {
-        const int cnt = min(u_end, (kvh + 1) * n_ch) - max(u_begin, kvh * n_ch);
+    consumer_sync();
+    for (int kvh = ar.u_begin / ar.n_ch; kvh <= (ar.u_end - 1) / ar.n_ch; ++kvh) {
+        const int cnt = min(ar.u_end, (kvh + 1) * ar.n_ch) - max(ar.u_begin, kvh * ar.n_ch);
         if (tid == 0) {
             const unsigned prev = atomicAdd(&a.counters[kvh], (unsigned)cnt);
-            s_last = prev + (unsigned)cnt == (unsigned)n_ch;
+            s_last = prev + (unsigned)cnt == (unsigned)ar.n_ch;
         }
-        __syncthreads();
+        consumer_sync();
         if (s_last) {
             __threadfence();
             const float* part = a.part + (size_t)kvh * a.n_chunks * NV * part_v;
             // row m uses chunks 0 .. (pos0 + m) / 64
-            for (int v = wk ? warp : NV; v < NV; v += kAttnThreads / 32) {
+            for (int v = warp; v < NV; v += kConsumers / 32) {
                 const int m = v / G, gi = v - m * G;
                 const int nch = (pos0 + m) / kAttnChunk + 1;
                 float mx = -INFINITY;
-                for (int cc = lane; cc < nch; cc += 32) mx = fmaxf(mx, __ldcg(part + ((size_t)cc * NV + v) * part_v + HD));
+                for (int cc = lane; cc < nch; cc += 32)
+                    mx = fmaxf(mx, __ldcg(part + ((size_t)cc * NV + v) * part_v + HD));
                 mx = warp_max(mx);
                 float lp = 0.f;
                 for (int cc = lane; cc < nch; cc += 32) {
-                    const float* pp = part + ((size_t)cc * NV + v) * part_v;
-                    const float mc = __ldcg(pp + HD);
-                    if (mc != -INFINITY) lp += expf(mc - mx) * __ldcg(pp + HD + 1);
+                    const float* pp2 = part + ((size_t)cc * NV + v) * part_v;
+                    const float mc = __ldcg(pp2 + HD);
+                    if (mc != -INFINITY) lp += expf(mc - mx) * __ldcg(pp2 + HD + 1);
                 }
                 const float inv = 1.f / warp_sum(lp);
                 float o[EPL];
@@ -785,11 +834,11 @@ __device__ void attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem)
                 for (int e = 0; e < EPL; ++e) o[e] = 0.f;
 #pragma unroll 4
                 for (int cc = 0; cc < nch; ++cc) {
-                    const float* pp = part + ((size_t)cc * NV + v) * part_v;
-                    const float mc = __ldcg(pp + HD);
+                    const float* pp2 = part + ((size_t)cc * NV + v) * part_v;
+                    const float mc = __ldcg(pp2 + HD);
                     const float f = mc == -INFINITY ? 0.f : expf(mc - mx);  // empty chunks hold o = 0
 #pragma unroll
-                    for (int e = 0; e < EPL; ++e) o[e] += f * __ldcg(pp + lane * EPL + e);
+                    for (int e = 0; e < EPL; ++e) o[e] += f * __ldcg(pp2 + lane * EPL + e);
                 }
                 const size_t at = (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + lane * EPL;
 #pragma unroll
@@ -802,8 +851,9 @@ __device__ void attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem)
             }
             if (tid == 0) a.counters[kvh] = 0u;
         }
-        __syncthreads();
+        consumer_sync();
     }
+    return ok;
 }
 
 // ---------------------------------------------------------------------------
@@ -911,7 +961,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
                             (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr, ct);
         } else {
             if (type == OP_EMBED) embed_op(p, pos0);
-            else attn_op<HD>(op.at, p.M, pos0, smem);
+            else ok = attn_op<R, HD>(op.at, p.M, pos0, smem, pp, p.err);
         }
         if (ct && threadIdx.x == 0) ct[3] = globaltimer();
         prefetched = false;
@@ -966,9 +1016,6 @@ size_t forward_smem_bytes(int M) {
     return R == 1 ? GemmSmem<1>::BYTES : (R == 8 ? GemmSmem<8>::BYTES : GemmSmem<16>::BYTES);
 }
 
-size_t attention_smem_bytes(int head_dim, int group, int M) {
-    return (size_t)kAttnBufs * 2 * kAttnChunk * (head_dim * 2 + 16) + (size_t)group * M * (head_dim + kAttnChunk) * 4;
-}
 
 int forward_configure() {
     int e = 0;

@@ -99,8 +99,11 @@ struct GemmArgs {
 // ---------------------------------------------------------------------------
 struct AttnArgs {
     const float* q;      // [M][H*hd]
-    const f16* k_cache;  // [Hkv][max_seq][hd] fp16
-    const f16* v_cache;
+    // TMA maps of the whole K / V cache viewed as {hd, max_seq, L * Hkv} fp16,
+    // box {64, 64, 1}, 128-byte swizzle; this layer's KV head kvh is z = kv_z0 + kvh
+    const void* tm_k;
+    const void* tm_v;
+    int kv_z0;
     bf16* out_hi;        // [M][H*hd] output planes: hi = rn(o), lo = rn(o - hi)
     bf16* out_lo;
     float* part;         // [Hkv][n_chunks][G*M][hd + 2]
@@ -152,7 +155,6 @@ struct FwdParams {
 
 int forward_configure();
 size_t forward_smem_bytes(int M);
-size_t attention_smem_bytes(int head_dim, int group, int M);
 int launch_forward(const FwdParams& p, int head_dim, int grid, cudaStream_t s);
 
 // sets the thread's ssd_last_error() message and returns code
