@@ -201,6 +201,12 @@ __device__ __forceinline__ void prefetch_tmap(const void* tmap) {
 // narrow layout (K % 64 != 0, one copy per 64-wide k-box):
 //   weights: [k-box 4][row 64][64]: kbox * 8 KB + r * 128
 //   inputs : [k-box 4][max(2R, 8) rows][64]: kbox * XKB + p * 128
+// attention: 64-position chunks per segment (one ring stage each).  Segments
+// are absolute, so a row's softmax partials do not depend on M; two chunks
+// per segment balance ~150 CTAs well at LLaMA-2 KV-head counts and contexts
+// and keep the final combine short.
+constexpr int kAttnSegChunks = 2;
+
 // Attention unit in a stage: K rows of the 64-position chunk at 0 (dims 0-63,
 // then 64-127 at 8 KB), V rows at 16 KB; position t, 16-byte chunk c of a
 // 64-dim box at box + t * 128 + ((c ^ (t & 7)) << 4).
@@ -215,13 +221,13 @@ struct GemmSmem {
     static constexpr int XB = XR * ROWB;         // = 4 * XKB
     static constexpr int STAGE = WB + XB;
     static constexpr int RC = NT * 8;
+    static constexpr int VG = 16;  // attention: query vectors per pass over a staged segment
     static constexpr int S = 4;  // ring depth (5 or 6 stages, where they fit, measured no faster)
-    static constexpr int VG = 16;  // attention: query vectors per pass over a staged chunk
     static constexpr int RED = S * STAGE;                // [64][RC] floats
     static constexpr int YS = RED + kTileRows * RC * 4;  // [64][16] floats
-    static constexpr int ATT = RED;                      // [VG][128] q, [VG][64] scores
+    static constexpr int ATT = RED;                      // [VG][128] q, [VG][SEG] scores
     static constexpr int SCRATCH_GEMM = kTileRows * RC * 4 + kTileRows * 16 * 4;
-    static constexpr int SCRATCH_ATT = VG * 128 * 4 + VG * kAttnChunk * 4;
+    static constexpr int SCRATCH_ATT = VG * 128 * 4 + VG * kAttnSegChunks * kAttnChunk * 4;
     static constexpr size_t BYTES =
         1024 + (size_t)RED + (SCRATCH_GEMM > SCRATCH_ATT ? SCRATCH_GEMM : SCRATCH_ATT);
 };
@@ -629,81 +635,84 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 }
 
 // ---------------------------------------------------------------------------
-// attention op: units (KV head, 64-position chunk), through the TMA ring
+// attention op: items (KV head, 256-position segment), through the TMA ring
 // ---------------------------------------------------------------------------
-// Each CTA takes a contiguous run of units.  The producer thread requests the
-// K / V rows of each unit (TMA, 128-byte swizzle) into the ring's stages, so
-// the copies of the next units are in flight while one is computed, and after
-// its last unit it goes on to the next projection's weights.  Per unit, for
-// its G * M query vectors v (G query heads of the KV head, M rows), in passes
-// of up to VG vectors: scores (one thread per (v, position)), softmax
-// partial (one warp per v), P V (one thread per (v, dimension pair)); the
-// partial (o, max, sum) goes to global memory.  After its units, a CTA adds
-// its count to each KV head's counter; the last arrival combines the chunk
-// partials of that head in chunk order (flash-decoding style split of the
-// softmax over position chunks).  Every reduction has a fixed order that
-// depends only on the row's own position, not on M.
+// A segment is kAttnSegChunks absolute 64-position chunks; the producer thread
+// requests each chunk's K and V rows (TMA, 128-byte swizzle) into consecutive
+// ring stages, and after the CTA's last chunk it goes on to prefetch the next
+// projection's weights.  The consumers hold a segment's stages at once and,
+// for its G * M query vectors v (G query heads of the KV head, M rows), in
+// passes of up to VG vectors: scores (one thread per (v, position)), softmax
+// over the segment (one warp per v), P V (eight threads per (v, 4 dims),
+// interleaved positions, fixed shuffle tree); the partial (o, max, sum) of the segment goes to
+// global memory.  After its items, a CTA adds its count to each KV head's
+// counter; the last arrival combines the segment partials of that head in
+// segment order (flash-decoding style split of the softmax).  Every reduction
+// has a fixed order that depends only on the row's own position, not on M.
 struct AttnRange {
-    int n_ch, u_begin, u_end;
+    int n_ch, n_seg, i_begin, i_end;  // chunks, segments per KV head; this CTA's items
 };
 __device__ __forceinline__ AttnRange attn_range(const AttnArgs& a, int M, int pos0) {
+    constexpr int S = kAttnSegChunks;
     AttnRange r;
     r.n_ch = (pos0 + M + kAttnChunk - 1) / kAttnChunk;  // chunks holding any visible position
-    const long long U = (long long)a.n_kv_heads * r.n_ch, GR = gridDim.x;
-    r.u_begin = (int)((long long)blockIdx.x * U / GR);
-    r.u_end = (int)((long long)(blockIdx.x + 1) * U / GR);
+    r.n_seg = (r.n_ch + S - 1) / S;
+    const long long I = (long long)a.n_kv_heads * r.n_seg, GR = gridDim.x;
+    r.i_begin = (int)((long long)blockIdx.x * I / GR);
+    r.i_end = (int)((long long)(blockIdx.x + 1) * I / GR);
     return r;
 }
 
 // Returns false if a wait timed out (error recorded).
 template <int R, int HD>
-__device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem, Pipe& pp, int* err) {
+__device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem, Pipe& pp, int* err,
+                        unsigned long long* ct) {
     using L = GemmSmem<R>;
-    constexpr int S = L::S, VG = L::VG;
-    constexpr int EPL = HD / 32;  // output dims per lane in the combine
+    constexpr int S = L::S, VG = L::VG, SC = kAttnSegChunks, SP = SC * kAttnChunk;  // positions per segment
+    static_assert(SC <= S, "a segment's chunks are held in the ring at once");
     const int G = a.n_heads / a.n_kv_heads, NV = G * M;
     const AttnRange ar = attn_range(a, M, pos0);
 
     if (threadIdx.x >= kConsumers) {  // producer warp: one elected thread requests K / V
         if (threadIdx.x != kConsumers) return true;
-        if (ar.u_begin < ar.u_end) {
+        if (ar.i_begin < ar.i_end) {
             // K / V rows of this forward were stored by other CTAs (generic proxy)
             asm volatile("fence.proxy.async.global;" ::: "memory");
             prefetch_tmap(a.tm_k);
             prefetch_tmap(a.tm_v);
         }
-        for (int u = ar.u_begin; u < ar.u_end; ++u) {
-            const int i = u - ar.u_begin, s = i % S;
-            unsigned char* st = smem + s * L::STAGE;
-            const int kvh = u / ar.n_ch, t0 = (u - kvh * ar.n_ch) * kAttnChunk;
-            if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return false;
-            pp.pphase ^= 1u << s;
-            mbar_arrive_expect_tx(pp.full + s, 2u * (HD / 64) * 8192u);
+        int i = 0;  // ring position within the op
+        for (int it = ar.i_begin; it < ar.i_end; ++it) {
+            const int kvh = it / ar.n_seg, c0 = (it - kvh * ar.n_seg) * SC;
+            for (int c = c0; c < min(c0 + SC, ar.n_ch); ++c, ++i) {
+                const int s = i % S;
+                unsigned char* st = smem + s * L::STAGE;
+                if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return false;
+                pp.pphase ^= 1u << s;
+                mbar_arrive_expect_tx(pp.full + s, 2u * (HD / 64) * 8192u);
 #pragma unroll
-            for (int bx = 0; bx < HD / 64; ++bx) {
-                tma_load_3d(st + bx * 8192, a.tm_k, bx * 64, t0, a.kv_z0 + kvh, pp.full + s);
-                tma_load_3d(st + 16384 + bx * 8192, a.tm_v, bx * 64, t0, a.kv_z0 + kvh, pp.full + s);
+                for (int bx = 0; bx < HD / 64; ++bx) {
+                    tma_load_3d(st + bx * 8192, a.tm_k, bx * 64, c * kAttnChunk, a.kv_z0 + kvh, pp.full + s);
+                    tma_load_3d(st + 16384 + bx * 8192, a.tm_v, bx * 64, c * kAttnChunk, a.kv_z0 + kvh, pp.full + s);
+                }
             }
         }
         return true;
     }
 
     float* qs = reinterpret_cast<float*>(smem + L::ATT);  // [VG][HD]
-    float* sc = qs + VG * HD;                              // [VG][64] scores, then weights
-    __shared__ int s_last;
+    float* sc = qs + VG * HD;                              // [VG][SP] scores, then weights
+    __shared__ unsigned s_mask;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const size_t part_v = HD + 2;  // floats per partial: o[HD], max, sum
     int q_kvh = -1;
     bool ok = true;
+    int i = 0;  // ring position within the op
 
-    for (int u = ar.u_begin; u < ar.u_end; ++u) {
-        const int i = u - ar.u_begin, s = i % S;
-        const unsigned char* ks = smem + s * L::STAGE;
-        const unsigned char* vs = ks + 16384;
-        const int kvh = u / ar.n_ch, c = u - kvh * ar.n_ch, t0 = c * kAttnChunk;
-        float* part = a.part + (size_t)kvh * a.n_chunks * NV * part_v;
-        ok = mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err) && ok;
-        pp.cphase ^= 1u << s;
+    for (int it = ar.i_begin; it < ar.i_end; ++it) {
+        const int kvh = it / ar.n_seg, sg = it - kvh * ar.n_seg, t0 = sg * SP;
+        const int n_u = min(SC, ar.n_ch - sg * SC);  // chunks of this segment
+        float* part = a.part + ((size_t)kvh * a.n_chunks + sg) * NV * part_v;
         for (int v0 = 0; v0 < NV; v0 += VG) {
             const int nv = min(VG, NV - v0);
             if (kvh != q_kvh || NV > VG) {  // q of this pass (written by other CTAs: L2)
@@ -713,30 +722,39 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
                     qs[k] = __ldcg(a.q + (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e);
                 }
                 q_kvh = kvh;
-                consumer_sync();
             }
+            if (v0 == 0) {  // K / V of the segment (the q loads above overlap the wait)
+                for (int j = 0; j < n_u; ++j) {
+                    const int s = (i + j) % S;
+                    ok = mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err) && ok;
+                    pp.cphase ^= 1u << s;
+                }
+                if (ct && tid == 0 && it == ar.i_begin) ct[1] = globaltimer();
+            }
+            consumer_sync();
             // scores: thread per (v, t); row m sees positions <= pos0 + m
-            for (int k = tid; k < nv * kAttnChunk; k += kConsumers) {
-                const int vl = k / kAttnChunk, t = k - vl * kAttnChunk;
-                const int m = (v0 + vl) / G;
+            for (int k = tid; k < nv * SP; k += kConsumers) {
+                const int vl = k / SP, t = k - vl * SP;
+                const int m = (v0 + vl) / G, j = t / kAttnChunk, tt = t - j * kAttnChunk;
                 float dot = -INFINITY;
-                if (t0 + t <= pos0 + m) {
+                if (j < n_u && t0 + t <= pos0 + m) {
+                    const unsigned char* ks = smem + ((i + j) % S) * L::STAGE;
                     float d0 = 0.f, d1 = 0.f;
-                    const float* q = qs + vl * HD;
-                    const int sw = t & 7;
+                    const float4* q4 = reinterpret_cast<const float4*>(qs + vl * HD);
+                    const int sw = tt & 7;
 #pragma unroll
                     for (int bx = 0; bx < HD / 64; ++bx) {
 #pragma unroll
                         for (int cc = 0; cc < 8; ++cc) {
                             const uint4 kv =
-                                *reinterpret_cast<const uint4*>(ks + bx * 8192 + t * 128 + ((cc ^ sw) << 4));
-                            const float* qq = q + bx * 64 + cc * 8;
+                                *reinterpret_cast<const uint4*>(ks + bx * 8192 + tt * 128 + ((cc ^ sw) << 4));
+                            const float4 qa = q4[bx * 16 + cc * 2], qb = q4[bx * 16 + cc * 2 + 1];
                             const float2 k0 = f16x2(kv.x), k1 = f16x2(kv.y), k2 = f16x2(kv.z), k3 = f16x2(kv.w);
                             float& d = (cc & 1) ? d1 : d0;
-                            d += qq[0] * k0.x + qq[1] * k0.y;
-                            d += qq[2] * k1.x + qq[3] * k1.y;
-                            d += qq[4] * k2.x + qq[5] * k2.y;
-                            d += qq[6] * k3.x + qq[7] * k3.y;
+                            d += qa.x * k0.x + qa.y * k0.y;
+                            d += qa.z * k1.x + qa.w * k1.y;
+                            d += qb.x * k2.x + qb.y * k2.y;
+                            d += qb.z * k3.x + qb.w * k3.y;
                         }
                     }
                     dot = (d0 + d1) * a.scale;
@@ -745,111 +763,146 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
             }
             consumer_sync();
 
-            // softmax partial: warp per v (positions lane, lane + 32)
+            // softmax over the segment: warp per v, positions lane + 32 q
             for (int vl = warp; vl < nv; vl += kConsumers / 32) {
                 const int v = v0 + vl, m = v / G;
-                float* o = part + ((size_t)c * NV + v) * part_v;
-                float* sv = sc + vl * kAttnChunk;
-                if (pos0 + m < t0) {  // nothing visible in this chunk
-                    sv[lane] = sv[lane + 32] = 0.f;
+                float* o = part + (size_t)v * part_v;
+                float* sv = sc + vl * SP;
+                if (pos0 + m < t0) {  // nothing visible in this segment
+#pragma unroll
+                    for (int q = 0; q < SP / 32; ++q) sv[lane + 32 * q] = 0.f;
                     if (lane == 0) { o[HD] = -INFINITY; o[HD + 1] = 0.f; }
                     continue;
                 }
-                const float s0 = sv[lane], s1 = sv[lane + 32];
-                const float mx = warp_max(fmaxf(s0, s1));
-                const float p0 = s0 == -INFINITY ? 0.f : expf(s0 - mx);
-                const float p1 = s1 == -INFINITY ? 0.f : expf(s1 - mx);
-                const float l = warp_sum(p0 + p1);
-                sv[lane] = p0;
-                sv[lane + 32] = p1;
+                float mx = -INFINITY;
+#pragma unroll
+                for (int q = 0; q < SP / 32; ++q) mx = fmaxf(mx, sv[lane + 32 * q]);
+                mx = warp_max(mx);
+                float l = 0.f;
+#pragma unroll
+                for (int q = 0; q < SP / 32; ++q) {
+                    const float x = sv[lane + 32 * q];
+                    const float pq = x == -INFINITY ? 0.f : expf(x - mx);
+                    sv[lane + 32 * q] = pq;
+                    l += pq;
+                }
+                l = warp_sum(l);
                 if (lane == 0) { o[HD] = mx; o[HD + 1] = l; }
             }
             consumer_sync();
 
-            // P V: thread per (v, dimension pair), even and odd positions in
-            // two accumulator pairs, summed at the end
-            for (int k = tid; k < nv * (HD / 2); k += kConsumers) {
-                const int vl = k / (HD / 2), e2 = k - vl * (HD / 2);
+            // P V: eight threads per (v, 4 dims); thread g sums positions g, g + 8,
+            // ... in order (rows with distinct swizzle phases: no bank
+            // conflicts), then a fixed shuffle tree over the eight
+            for (int k = tid; k < nv * (HD / 4) * 8; k += kConsumers) {
+                const int g = k & 7, e4 = (k >> 3) % (HD / 4), vl = k / (2 * HD);
                 const int v = v0 + vl, m = v / G;
-                const int n_t = min(kAttnChunk, pos0 + m + 1 - t0);  // <= 0: nothing visible
-                const float* pv = sc + vl * kAttnChunk;
-                const int e = 2 * e2, bx = e >> 6, cc = (e & 63) >> 3, off = (e & 7) * 2;
-                const unsigned char* vb = vs + bx * 8192 + off;
-                float a0 = 0.f, a1 = 0.f, b0 = 0.f, b1 = 0.f;
-                int t = 0;
-                for (; t + 1 < n_t; t += 2) {
-                    const float2 va = f16x2(*reinterpret_cast<const uint32_t*>(vb + t * 128 + ((cc ^ (t & 7)) << 4)));
-                    const float2 vn =
-                        f16x2(*reinterpret_cast<const uint32_t*>(vb + (t + 1) * 128 + ((cc ^ ((t + 1) & 7)) << 4)));
-                    a0 += pv[t] * va.x;
-                    a1 += pv[t] * va.y;
-                    b0 += pv[t + 1] * vn.x;
-                    b1 += pv[t + 1] * vn.y;
+                const int e = 4 * e4, bx = e >> 6, cc = (e & 63) >> 3, off = (e & 7) * 2;
+                float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+                for (int j = 0; j < n_u; ++j) {
+                    const int n_t = min(kAttnChunk, pos0 + m + 1 - (t0 + j * kAttnChunk));  // <= 0: none
+                    const float* pv = sc + vl * SP + j * kAttnChunk;
+                    const unsigned char* vb = smem + ((i + j) % S) * L::STAGE + 16384 + bx * 8192 + off;
+#pragma unroll 4
+                    for (int t = g; t < n_t; t += 8) {
+                        const uint2 va = *reinterpret_cast<const uint2*>(vb + t * 128 + ((cc ^ (t & 7)) << 4));
+                        const float pa = pv[t];
+                        const float2 x0 = f16x2(va.x), x1 = f16x2(va.y);
+                        a0 += pa * x0.x;
+                        a1 += pa * x0.y;
+                        a2 += pa * x1.x;
+                        a3 += pa * x1.y;
+                    }
                 }
-                if (t < n_t) {
-                    const float2 va = f16x2(*reinterpret_cast<const uint32_t*>(vb + t * 128 + ((cc ^ (t & 7)) << 4)));
-                    a0 += pv[t] * va.x;
-                    a1 += pv[t] * va.y;
+#pragma unroll
+                for (int w = 1; w < 8; w <<= 1) {
+                    a0 += __shfl_xor_sync(0xffffffffu, a0, w);
+                    a1 += __shfl_xor_sync(0xffffffffu, a1, w);
+                    a2 += __shfl_xor_sync(0xffffffffu, a2, w);
+                    a3 += __shfl_xor_sync(0xffffffffu, a3, w);
                 }
-                float* o = part + ((size_t)c * NV + v) * part_v;
-                *reinterpret_cast<float2*>(o + e) = make_float2(a0 + b0, a1 + b1);
+                if (g == 0) {
+                    float* o = part + (size_t)v * part_v + e;
+                    *reinterpret_cast<float2*>(o) = make_float2(a0, a1);
+                    *reinterpret_cast<float2*>(o + 2) = make_float2(a2, a3);
+                }
             }
             consumer_sync();  // scores / q of this pass are free
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(pp.empty + s);  // the stage is free
+        if (lane == 0)
+            for (int j = 0; j < n_u; ++j) mbar_arrive(pp.empty + (i + j) % S);  // the stages are free
+        i += n_u;
     }
-    if (ar.u_begin >= ar.u_end) return ok;
+    if (ar.i_begin >= ar.i_end) return ok;
+    if (ct && tid == 0) {
+        ct[2] = globaltimer();
+        ct[6] = (unsigned long long)(ar.i_end - ar.i_begin);
+    }
 
-    // publish the partials; per KV head, the CTA that completes the count combines
+    // publish the partials; each KV head's count is completed by one CTA, which
+    // combines that head (all heads a CTA completes are combined in one pass)
     __threadfence();
     consumer_sync();
-    for (int kvh = ar.u_begin / ar.n_ch; kvh <= (ar.u_end - 1) / ar.n_ch; ++kvh) {
-        const int cnt = min(ar.u_end, (kvh + 1) * ar.n_ch) - max(ar.u_begin, kvh * ar.n_ch);
-        if (tid == 0) {
-            const unsigned prev = atomicAdd(&a.counters[kvh], (unsigned)cnt);
-            s_last = prev + (unsigned)cnt == (unsigned)ar.n_ch;
+    const int kv_lo = ar.i_begin / ar.n_seg, kv_hi = (ar.i_end - 1) / ar.n_seg;
+    for (int kb = kv_lo; kb <= kv_hi; kb += 32) {
+        const int nk = min(32, kv_hi - kb + 1);
+        if (warp == 0) {
+            bool last = false;
+            if (lane < nk) {
+                const int kvh = kb + lane;
+                const int cnt = min(ar.i_end, (kvh + 1) * ar.n_seg) - max(ar.i_begin, kvh * ar.n_seg);
+                const unsigned prev = atomicAdd(&a.counters[kvh], (unsigned)cnt);
+                last = prev + (unsigned)cnt == (unsigned)ar.n_seg;
+                if (last) a.counters[kvh] = 0u;  // no other CTA touches it again in this op
+            }
+            const unsigned mask = __ballot_sync(0xffffffffu, last);
+            if (lane == 0) s_mask = mask;
         }
         consumer_sync();
-        if (s_last) {
+        const int n_last = __popc(s_mask);
+        if (n_last) {
             __threadfence();
-            const float* part = a.part + (size_t)kvh * a.n_chunks * NV * part_v;
-            // row m uses chunks 0 .. (pos0 + m) / 64
-            for (int v = warp; v < NV; v += kConsumers / 32) {
+            // row m uses segments 0 .. (pos0 + m) / SP, summed in segment order;
+            // thread per (head, v, 4 dims): every load of a row is independent
+            for (int k = tid; k < n_last * NV * (HD / 4); k += kConsumers) {
+                const int hx = k / (NV * (HD / 4)), kk = k - hx * NV * (HD / 4);
+                unsigned mm = s_mask;  // the hx-th head this CTA completed
+                for (int r = 0; r < hx; ++r) mm &= mm - 1u;
+                const int kvh = kb + __ffs(mm) - 1;
+                const float* part = a.part + (size_t)kvh * a.n_chunks * NV * part_v;
+                const int v = kk / (HD / 4), e = (kk - v * (HD / 4)) * 4;
                 const int m = v / G, gi = v - m * G;
-                const int nch = (pos0 + m) / kAttnChunk + 1;
+                const int nsg = (pos0 + m) / SP + 1;
+                const float* pv = part + (size_t)v * part_v;
+                const size_t qs_stride = (size_t)NV * part_v;
                 float mx = -INFINITY;
-                for (int cc = lane; cc < nch; cc += 32)
-                    mx = fmaxf(mx, __ldcg(part + ((size_t)cc * NV + v) * part_v + HD));
-                mx = warp_max(mx);
-                float lp = 0.f;
-                for (int cc = lane; cc < nch; cc += 32) {
-                    const float* pp2 = part + ((size_t)cc * NV + v) * part_v;
-                    const float mc = __ldcg(pp2 + HD);
-                    if (mc != -INFINITY) lp += expf(mc - mx) * __ldcg(pp2 + HD + 1);
+#pragma unroll 8
+                for (int q = 0; q < nsg; ++q) mx = fmaxf(mx, __ldcg(pv + q * qs_stride + HD));
+                float l = 0.f, o0 = 0.f, o1 = 0.f, o2 = 0.f, o3 = 0.f;
+#pragma unroll 8
+                for (int q = 0; q < nsg; ++q) {
+                    const float* pq = pv + q * qs_stride;
+                    const float mq = __ldcg(pq + HD);
+                    const float f = mq == -INFINITY ? 0.f : expf(mq - mx);  // empty segments hold o = 0
+                    const float2 oa = __ldcg(reinterpret_cast<const float2*>(pq + e));
+                    const float2 ob = __ldcg(reinterpret_cast<const float2*>(pq + e + 2));
+                    l += f * __ldcg(pq + HD + 1);
+                    o0 += f * oa.x;
+                    o1 += f * oa.y;
+                    o2 += f * ob.x;
+                    o3 += f * ob.y;
                 }
-                const float inv = 1.f / warp_sum(lp);
-                float o[EPL];
+                const float inv = 1.f / l;
+                const size_t at = (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e;
+                const float val[4] = {o0 * inv, o1 * inv, o2 * inv, o3 * inv};
 #pragma unroll
-                for (int e = 0; e < EPL; ++e) o[e] = 0.f;
-#pragma unroll 4
-                for (int cc = 0; cc < nch; ++cc) {
-                    const float* pp2 = part + ((size_t)cc * NV + v) * part_v;
-                    const float mc = __ldcg(pp2 + HD);
-                    const float f = mc == -INFINITY ? 0.f : expf(mc - mx);  // empty chunks hold o = 0
-#pragma unroll
-                    for (int e = 0; e < EPL; ++e) o[e] += f * __ldcg(pp2 + lane * EPL + e);
-                }
-                const size_t at = (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + lane * EPL;
-#pragma unroll
-                for (int e = 0; e < EPL; ++e) {
-                    const float val = o[e] * inv;
-                    const bf16 vh = __float2bfloat16_rn(val);
-                    a.out_hi[at + e] = vh;
-                    a.out_lo[at + e] = __float2bfloat16_rn(val - __bfloat162float(vh));
+                for (int x = 0; x < 4; ++x) {
+                    const bf16 vh = __float2bfloat16_rn(val[x]);
+                    a.out_hi[at + x] = vh;
+                    a.out_lo[at + x] = __float2bfloat16_rn(val[x] - __bfloat162float(vh));
                 }
             }
-            if (tid == 0) a.counters[kvh] = 0u;
         }
         consumer_sync();
     }
@@ -961,7 +1014,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
                             (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr, ct);
         } else {
             if (type == OP_EMBED) embed_op(p, pos0);
-            else ok = attn_op<R, HD>(op.at, p.M, pos0, smem, pp, p.err);
+            else ok = attn_op<R, HD>(op.at, p.M, pos0, smem, pp, p.err, ct);
         }
         if (ct && threadIdx.x == 0) ct[3] = globaltimer();
         prefetched = false;
