@@ -175,15 +175,16 @@ const bf16* next_norm(const ssd_handle* h, int s, bool draft) {
 
 // ---------------------------------------------------------------------------
 // TMA descriptors.  Index layout: layer l's wq wk wv wo w_gate w_up w_down at
-// 7l + 0..6, lm_head at 7L, then the input-plane maps at 7L + 1 + buf * 3 + cls
+// 7l + 0..6, lm_head at 7L, then the input-plane maps at 7L + 1 + buf * 4 + cls
 // with buf 0 = normalised rows (K = d), 1 = attention output (K = H*hd),
-// 2 = SwiGLU output (K = ffn) and cls = rows per plane 1 | 8 | 16.
+// 2 = SwiGLU output (K = ffn) and cls = rows per plane 1 | 8 | 12 | 16, then the
+// K and V cache maps.
 // ---------------------------------------------------------------------------
 size_t trace_words(const ssd_handle* h) { return (size_t)kTraceCtas + 8 * (size_t)h->n_sms; }
 
 int tmap_weight(int l, int which) { return 7 * l + which; }
-int tmap_x(const ssd_handle* h, int buf, int cls) { return 7 * h->cfg.n_layers + 1 + buf * 3 + cls; }
-int tmap_kv(const ssd_handle* h, int v) { return 7 * h->cfg.n_layers + 10 + v; }
+int tmap_x(const ssd_handle* h, int buf, int cls) { return 7 * h->cfg.n_layers + 1 + buf * kPlaneClasses + cls; }
+int tmap_kv(const ssd_handle* h, int v) { return 7 * h->cfg.n_layers + 1 + 3 * kPlaneClasses + v; }
 
 // Checks the TMA rules and encodes a 16-bit tensor map with 64-element (128-byte)
 // inner boxes, 128-byte swizzle, zero fill out of range: base 16-byte aligned,
@@ -255,9 +256,9 @@ int build_tmaps(ssd_handle* h) {
     if (!rc) rc = encode_weight(enc, &maps[7 * L], h->lm_head, d, c.vocab);
     const bf16* planes[3] = {h->xn_hi, h->at_hi, h->ac_hi};
     const int widths[3] = {d, qd, c.ffn};
-    const int rows[3] = {1, 8, 16};
+    const int rows[kPlaneClasses] = {1, 8, 12, 16};
     for (int b = 0; b < 3 && !rc; ++b)
-        for (int cls = 0; cls < 3 && !rc; ++cls)
+        for (int cls = 0; cls < kPlaneClasses && !rc; ++cls)
             rc = encode_planes(enc, &maps[tmap_x(h, b, cls)], planes[b], widths[b], rows[cls]);
     // K / V cache [L][Hkv][max_seq][hd] fp16 as {hd, max_seq, L * Hkv}, box 64 dims x 64 positions
     for (int v = 0; v < 2 && !rc; ++v) {
@@ -274,7 +275,7 @@ int build_tmaps(ssd_handle* h) {
 }
 
 void set_x_maps(const ssd_handle* h, GemmArgs& a, int buf) {
-    for (int cls = 0; cls < 3; ++cls) a.tm_x[cls] = h->tmaps + tmap_x(h, buf, cls);
+    for (int cls = 0; cls < kPlaneClasses; ++cls) a.tm_x[cls] = h->tmaps + tmap_x(h, buf, cls);
 }
 
 // One projection op: fills the fields every projection shares.
@@ -662,7 +663,7 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
         return bail(rc);
     h->max_ops = 2 + 5 * L;
     if (h->max_ops + 1 > 1024) return bail(fail(SSD_ERR_INVALID_ARG, "too many layers (at most 204)"));
-    h->n_tmaps = 7 * L + 1 + 9 + 2;
+    h->n_tmaps = 7 * L + 1 + 3 * kPlaneClasses + 2;
     if ((rc = dalloc(h, &h->tmaps, (size_t)h->n_tmaps, &B)) ||
         (rc = dalloc(h, &h->ops_full, (size_t)h->max_ops, &B)) ||
         (rc = dalloc(h, &h->ops_draft, (size_t)h->max_ops, &B)) ||

@@ -212,6 +212,9 @@ constexpr int kAttnSegChunks = 2;
 // 64-dim box at box + t * 128 + ((c ^ (t & 7)) << 4).
 // After the ring: the consumers' scratch - split-K reduction buffers of a
 // projection, or (same bytes: one op at a time) q / scores of attention.
+// index of the input-plane tensor map of R rows
+__host__ __device__ constexpr int plane_cls(int R) { return R == 1 ? 0 : (R == 8 ? 1 : (R == 12 ? 2 : 3)); }
+
 template <int R>
 struct GemmSmem {
     static constexpr int NT = (2 * R + 7) / 8;   // n8 MMA tiles: 1 | 2 | 4
@@ -309,7 +312,7 @@ template <int R>
 __device__ __forceinline__ void tma_inputs(const GemmArgs& a, int u, unsigned char* st, uint64_t* bar) {
     using L = GemmSmem<R>;
     const int k0 = (u % a.n_chunks) * KC;
-    const int cls = R == 1 ? 0 : (R == 8 ? 1 : 2);
+    const int cls = plane_cls(R);
     unsigned char* xs = st + L::WB;
     if (a.wide) {
         mbar_arrive_expect_tx(bar, 4u * 2u * (unsigned)R * 128u);
@@ -341,7 +344,7 @@ __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, P
     bool ok = true;
     if (threadIdx.x == kConsumers) {
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        prefetch_tmap(a.tm_x[R == 1 ? 0 : (R == 8 ? 1 : 2)]);
+        prefetch_tmap(a.tm_x[plane_cls(R)]);
         for (int s = 0; s < S && s < n_my && ok; ++s) {
             ok = mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err);
             if (!ok) break;
@@ -1066,7 +1069,8 @@ int configure_fwd() {
 
 size_t forward_smem_bytes(int M) {
     const int R = fwd_plane_rows(M);
-    return R == 1 ? GemmSmem<1>::BYTES : (R == 8 ? GemmSmem<8>::BYTES : GemmSmem<16>::BYTES);
+    return R == 1 ? GemmSmem<1>::BYTES
+                  : (R == 8 ? GemmSmem<8>::BYTES : (R == 12 ? GemmSmem<12>::BYTES : GemmSmem<16>::BYTES));
 }
 
 
@@ -1074,9 +1078,11 @@ int forward_configure() {
     int e = 0;
     e = e ? e : configure_fwd<1, 64>();
     e = e ? e : configure_fwd<8, 64>();
+    e = e ? e : configure_fwd<12, 64>();
     e = e ? e : configure_fwd<16, 64>();
     e = e ? e : configure_fwd<1, 128>();
     e = e ? e : configure_fwd<8, 128>();
+    e = e ? e : configure_fwd<12, 128>();
     e = e ? e : configure_fwd<16, 128>();
     return e;
 }
@@ -1084,9 +1090,13 @@ int forward_configure() {
 int launch_forward(const FwdParams& p, int head_dim, int grid, cudaStream_t s) {
     const int R = fwd_plane_rows(p.M);
     if (head_dim == 128)
-        return R == 1 ? launch_fwd<1, 128>(p, grid, s) : (R == 8 ? launch_fwd<8, 128>(p, grid, s) : launch_fwd<16, 128>(p, grid, s));
+        return R == 1 ? launch_fwd<1, 128>(p, grid, s)
+             : R == 8 ? launch_fwd<8, 128>(p, grid, s)
+             : R == 12 ? launch_fwd<12, 128>(p, grid, s) : launch_fwd<16, 128>(p, grid, s);
     if (head_dim == 64)
-        return R == 1 ? launch_fwd<1, 64>(p, grid, s) : (R == 8 ? launch_fwd<8, 64>(p, grid, s) : launch_fwd<16, 64>(p, grid, s));
+        return R == 1 ? launch_fwd<1, 64>(p, grid, s)
+             : R == 8 ? launch_fwd<8, 64>(p, grid, s)
+             : R == 12 ? launch_fwd<12, 64>(p, grid, s) : launch_fwd<16, 64>(p, grid, s);
     return (int)cudaErrorInvalidValue;
 }
 

@@ -90,7 +90,7 @@ struct GemmArgs {
     // 64-wide k-box.
     int wide;
     const void* tm_w[3];  // w0, w1, w2
-    const void* tm_x[3];  // input planes for R = 1 | 8 | 16
+    const void* tm_x[4];  // input planes for R = 1 | 8 | 12 | 16
 };
 
 // ---------------------------------------------------------------------------
@@ -165,7 +165,9 @@ int gemm_configure();
 int launch_gemm(int epi, const GemmArgs& a, cudaStream_t s);
 size_t gemm_smem_bytes(int kc, int M);
 constexpr int gemm_half_rows(int M) { return M <= 8 ? 8 : 16; }  // padded rows of x_hi (and of x_lo)
-constexpr int fwd_plane_rows(int M) { return M == 1 ? 1 : (M <= 8 ? 8 : 16); }  // R of the forward kernel
+// R of the forward kernel: input-plane rows per op (1 | 8 | 12 | 16)
+constexpr int fwd_plane_rows(int M) { return M == 1 ? 1 : (M <= 8 ? 8 : (M <= 12 ? 12 : 16)); }
+constexpr int kPlaneClasses = 4;
 
 
 
