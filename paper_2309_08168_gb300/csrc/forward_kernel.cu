@@ -666,10 +666,55 @@ __device__ __forceinline__ AttnRange attn_range(const AttnArgs& a, int M, int po
     return r;
 }
 
-// Returns false if a wait timed out (error recorded).
+// Producer thread: requests K / V of this CTA's chunks at ring positions
+// [i_from, i_limit), in item order; with old_only it stops at the first chunk
+// holding rows this forward writes (those need the q/k/v op to be finished).
+// Returns the ring position reached, or -1 if a wait timed out.
+template <int R, int HD>
+__device__ int attn_produce(const AttnArgs& a, const AttnRange& ar, int pos0, unsigned char* smem, Pipe& pp,
+                            int* err, int i_from, int i_limit, bool old_only) {
+    using L = GemmSmem<R>;
+    constexpr int S = L::S, SC = kAttnSegChunks;
+    int i = 0;
+    for (int it = ar.i_begin; it < ar.i_end; ++it) {
+        const int kvh = it / ar.n_seg, c0 = (it - kvh * ar.n_seg) * SC;
+        for (int c = c0; c < min(c0 + SC, ar.n_ch); ++c, ++i) {
+            if (i < i_from) continue;
+            if (i >= i_limit || (old_only && (c + 1) * kAttnChunk > pos0)) return i;
+            const int s = i % S;
+            unsigned char* st = smem + s * L::STAGE;
+            if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return -1;
+            pp.pphase ^= 1u << s;
+            mbar_arrive_expect_tx(pp.full + s, 2u * (HD / 64) * 8192u);
+#pragma unroll
+            for (int bx = 0; bx < HD / 64; ++bx) {
+                tma_load_3d(st + bx * 8192, a.tm_k, bx * 64, c * kAttnChunk, a.kv_z0 + kvh, pp.full + s);
+                tma_load_3d(st + 16384 + bx * 8192, a.tm_v, bx * 64, c * kAttnChunk, a.kv_z0 + kvh, pp.full + s);
+            }
+        }
+    }
+    return i;
+}
+
+// Before the grid barrier ahead of an attention op: the producer requests the
+// K / V chunks of its first ring stages that hold only rows of earlier
+// forwards.  Returns how many (0 for other threads, -1 on a timeout).
+template <int R, int HD>
+__device__ int attn_prefetch(const AttnArgs& a, int M, int pos0, unsigned char* smem, Pipe& pp, int* err) {
+    if (threadIdx.x != kConsumers) return 0;
+    const AttnRange ar = attn_range(a, M, pos0);
+    if (ar.i_begin < ar.i_end) {
+        prefetch_tmap(a.tm_k);
+        prefetch_tmap(a.tm_v);
+    }
+    return attn_produce<R, HD>(a, ar, pos0, smem, pp, err, 0, GemmSmem<R>::S, true);
+}
+
+// Returns false if a wait timed out (error recorded).  pre: ring positions the
+// producer already filled before the grid barrier (attn_prefetch).
 template <int R, int HD>
 __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem, Pipe& pp, int* err,
-                        unsigned long long* ct) {
+                        unsigned long long* ct, int pre) {
     using L = GemmSmem<R>;
     constexpr int S = L::S, VG = L::VG, SC = kAttnSegChunks, SP = SC * kAttnChunk;  // positions per segment
     static_assert(SC <= S, "a segment's chunks are held in the ring at once");
@@ -678,29 +723,9 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
 
     if (threadIdx.x >= kConsumers) {  // producer warp: one elected thread requests K / V
         if (threadIdx.x != kConsumers) return true;
-        if (ar.i_begin < ar.i_end) {
-            // K / V rows of this forward were stored by other CTAs (generic proxy)
-            asm volatile("fence.proxy.async.global;" ::: "memory");
-            prefetch_tmap(a.tm_k);
-            prefetch_tmap(a.tm_v);
-        }
-        int i = 0;  // ring position within the op
-        for (int it = ar.i_begin; it < ar.i_end; ++it) {
-            const int kvh = it / ar.n_seg, c0 = (it - kvh * ar.n_seg) * SC;
-            for (int c = c0; c < min(c0 + SC, ar.n_ch); ++c, ++i) {
-                const int s = i % S;
-                unsigned char* st = smem + s * L::STAGE;
-                if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return false;
-                pp.pphase ^= 1u << s;
-                mbar_arrive_expect_tx(pp.full + s, 2u * (HD / 64) * 8192u);
-#pragma unroll
-                for (int bx = 0; bx < HD / 64; ++bx) {
-                    tma_load_3d(st + bx * 8192, a.tm_k, bx * 64, c * kAttnChunk, a.kv_z0 + kvh, pp.full + s);
-                    tma_load_3d(st + 16384 + bx * 8192, a.tm_v, bx * 64, c * kAttnChunk, a.kv_z0 + kvh, pp.full + s);
-                }
-            }
-        }
-        return true;
+        // K / V rows of this forward were stored by other CTAs (generic proxy)
+        if (ar.i_begin < ar.i_end) asm volatile("fence.proxy.async.global;" ::: "memory");
+        return attn_produce<R, HD>(a, ar, pos0, smem, pp, err, pre, 1 << 30, false) >= 0;
     }
 
     float* qs = reinterpret_cast<float*>(smem + L::ATT);  // [VG][HD]
@@ -999,6 +1024,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
     unsigned target = 0;
     Pipe pp{full, empty, 0u, 0u};
     bool prefetched = false;
+    int attn_pre = 0;  // producer: K / V chunks of the next attention op requested early
     copy_op(p.ops, s_op);
     for (int o = 0; o < p.n_ops; ++o) {
         const FwdOp& op = s_op[o & 1];
@@ -1017,13 +1043,17 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
                             (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr, ct);
         } else {
             if (type == OP_EMBED) embed_op(p, pos0);
-            else ok = attn_op<R, HD>(op.at, p.M, pos0, smem, pp, p.err, ct);
+            else ok = attn_op<R, HD>(op.at, p.M, pos0, smem, pp, p.err, ct, attn_pre);
         }
         if (ct && threadIdx.x == 0) ct[3] = globaltimer();
         prefetched = false;
+        attn_pre = 0;
         if (nx && ok && is_gemm(nx->type)) {
             ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err);
             prefetched = true;
+        } else if (nx && ok && nx->type == OP_ATTN) {
+            attn_pre = attn_prefetch<R, HD>(nx->at, p.M, pos0, smem, pp, p.err);
+            ok = attn_pre >= 0;
         }
         if (!ok) s_fail = 1;
         __syncthreads();
