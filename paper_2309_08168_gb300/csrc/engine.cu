@@ -730,6 +730,10 @@ int ssd_prefill(ssd_handle* h, const int32_t* prompt, int n_prompt) {
     CUDA_TRY(cudaSetDevice(h->device), "set device");
     h->prefilled = false;
     CUDA_TRY(cudaMemsetAsync(&h->st->err, 0, sizeof(int), h->stream), "error flag reset");
+    // arrival counters are left at zero by every completed op; after a timed-out
+    // forward they may not be, so a new prompt starts from clean counters
+    CUDA_TRY(cudaMemsetAsync(h->counters, 0, ((size_t)h->gemm_counters + h->cfg.n_kv_heads) * sizeof(unsigned),
+                             h->stream), "counter reset");
     if (n_prompt > 1)
         CUDA_TRY(cudaMemcpyAsync(h->tok, prompt, sizeof(int) * (n_prompt - 1), cudaMemcpyHostToDevice, h->stream),
                  "prompt upload");
@@ -742,7 +746,7 @@ int ssd_prefill(ssd_handle* h, const int32_t* prompt, int n_prompt) {
     {
         int derr = 0;
         CUDA_TRY(cudaMemcpy(&derr, &h->st->err, sizeof(int), cudaMemcpyDeviceToHost), "error flag");
-        if (derr == kDevErrTimeout) return fail(SSD_ERR_TIMEOUT, "a grid barrier of the forward kernel timed out");
+        if (derr == kDevErrTimeout) return fail(SSD_ERR_TIMEOUT, "a wait of the forward kernel timed out");
     }
 #ifdef SSD_CHECKED
     {

@@ -94,6 +94,27 @@ __device__ bool grid_barrier(unsigned* bar, unsigned target, int* err) {
     return s_ok != 0;
 }
 
+// fire-and-forget release increment (publishes this thread's earlier stores)
+__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Bounded wait until *c >= target (acquire); false (timeout recorded) after
+// kBarrierTimeoutNs or when another CTA already recorded an error.
+__device__ bool wait_count(const unsigned* c, unsigned target, int* err) {
+    if (ld_acquire(c) >= target) return true;
+    const unsigned long long t0 = globaltimer();
+    for (;;) {
+        __nanosleep(32);
+        if (ld_acquire(c) >= target) return true;
+        if (*(volatile int*)err) return false;
+        if (globaltimer() - t0 > kBarrierTimeoutNs) {
+            atomicCAS(err, 0, kDevErrTimeout);
+            return false;
+        }
+    }
+}
+
 __device__ __forceinline__ int unit_owner(long long u, long long U, long long G) {
     return (int)(((u + 1) * G + U - 1) / U - 1);
 }
@@ -147,12 +168,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, unsigned parity) {
         : "memory");
     return ok != 0;
 }
-// bounded wait: false (error recorded) after kWaitTimeoutNs
+// bounded wait: false after kWaitTimeoutNs (timeout recorded), or once it has
+// waited 20 us while another thread has already recorded an error
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity, int* err) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = globaltimer();
     while (!mbar_try_wait(bar, parity)) {
-        if (globaltimer() - t0 > kWaitTimeoutNs) {
+        const unsigned long long dt = globaltimer() - t0;
+        if (dt > 20000ull && *(volatile int*)err) return false;
+        if (dt > kWaitTimeoutNs) {
             atomicCAS(err, 0, kDevErrTimeout);
             return false;
         }
@@ -370,7 +394,7 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
     constexpr int S = L::S;
     float* red = reinterpret_cast<float*>(smem + L::RED);  // [64][RC]
     float* ys = reinterpret_cast<float*>(smem + L::YS);    // [64][16]
-    __shared__ int s_last;
+    bool ok = true;
 
     const long long U = a.n_units, G = op_ctas(U);
     const int b = blockIdx.x;
@@ -425,7 +449,9 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         const int s = i % S;
         const unsigned char* w_s = smem + s * L::STAGE;
         const unsigned char* x_s = w_s + L::WB;
-        if (!mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err)) return false;
+        // a failed wait leaves garbage in the stage: carry on (every consumer
+        // must reach every consumer barrier), the error is reported
+        ok = mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err) && ok;
         pp.cphase ^= 1u << s;
         if (threadIdx.x == 0) {
             if (ut && i < 64) ut[i * 4 + 1] = globaltimer();
@@ -507,45 +533,51 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         // RESID: this tile's residual h (written by earlier ops: L2), loaded
         // before the split-K exchange so its latency overlaps it
         constexpr int HJ = kMaxRows * kTileRows / kGemmThreads;
-        float hpre[HJ];
+        float hpre[HJ], gpre[HJ];
         if (epi == EPI_RESID) {
 #pragma unroll
             for (int j = 0; j < HJ; ++j) {
                 const int idx = threadIdx.x + j * kGemmThreads;
                 const int m = idx / kTileRows, n = tile * kTileRows + (idx - m * kTileRows);
-                hpre[j] = (idx < M * kTileRows && n < a.N) ? __ldcg(a.out_f32 + (size_t)m * a.ldo + n) : 0.f;
+                const bool in = idx < M * kTileRows && n < a.N;
+                hpre[j] = in ? __ldcg(a.out_f32 + (size_t)m * a.ldo + n) : 0.f;
+                gpre[j] = (in && a.g_next) ? __bfloat162float(a.g_next[n]) : 0.f;
             }
         }
 
-        // segments of other CTAs: the last one to arrive sums all in order
+        // split-K: the CTA holding the tile's first chunks (its segment ends
+        // last, at the end of that CTA's range) finalises; the others publish
+        // their partial and move on.  The sum is in segment order.
         const long long u_first = (long long)tile * a.n_chunks;
         const int seg0 = unit_owner(u_first, U, G);
         const int nseg = unit_owner(u_first + a.n_chunks - 1, U, G) - seg0 + 1;
         if (nseg > 1) {
             float* slots = a.partial + (size_t)tile * a.n_chunks * kMaxRows * kTileRows;
-            float* mine = slots + (size_t)(b - seg0) * kMaxRows * kTileRows;
-            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
-                const int m = idx / kTileRows, r = idx - m * kTileRows;
-                mine[m * kTileRows + r] = ys[r * 16 + m];
+            if (b != seg0) {
+                float* mine = slots + (size_t)(b - seg0) * kMaxRows * kTileRows;
+                for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+                    const int m = idx / kTileRows, r = idx - m * kTileRows;
+                    mine[m * kTileRows + r] = ys[r * 16 + m];
+                }
+                __threadfence();
+                consumer_sync();
+                if (threadIdx.x == 0) red_release_add(&a.counters[tile], 1u);
+                continue;
             }
-            __threadfence();
-            consumer_sync();
+            // the other segments come from later CTAs, which never wait on this one
             if (threadIdx.x == 0) {
-                const unsigned prev = atomicAdd(&a.counters[tile], 1u);
-                s_last = prev == (unsigned)(nseg - 1);
+                if (!wait_count(&a.counters[tile], (unsigned)(nseg - 1), err)) ok = false;
+                a.counters[tile] = 0u;  // every other segment has been counted
             }
             consumer_sync();
-            if (!s_last) continue;
-            __threadfence();
             for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
                 const int m = idx / kTileRows, r = idx - m * kTileRows;
                 const float* p = slots + m * kTileRows + r;
-                float sum = __ldcg(p);
+                float sum = ys[r * 16 + m];
 #pragma unroll 4
                 for (int sg = 1; sg < nseg; ++sg) sum += __ldcg(p + (size_t)sg * kMaxRows * kTileRows);
                 ys[r * 16 + m] = sum;
             }
-            if (threadIdx.x == 0) a.counters[tile] = 0u;
             consumer_sync();
         }
 
@@ -569,7 +601,7 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
                     hv = hpre[j] + ys[r * 16 + m];
                     *o = hv;
                     if (a.g_next) {
-                        const float z = hv * __bfloat162float(a.g_next[n]);
+                        const float z = hv * gpre[j];
                         const bf16 zh = __float2bfloat16_rn(z);
                         a.xo_hi[(size_t)m * a.N + n] = zh;
                         a.xo_lo[(size_t)m * a.N + n] = __float2bfloat16_rn(z - __bfloat162float(zh));
@@ -634,7 +666,7 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         if (ut && i < 64 && threadIdx.x == 0) ut[i * 4 + 3] = globaltimer();
     }
     consumer_sync();
-    return true;
+    return ok;
 }
 
 // ---------------------------------------------------------------------------
