@@ -678,7 +678,7 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 // projection's weights.  The consumers hold a segment's stages at once and,
 // for its G * M query vectors v (G query heads of the KV head, M rows), in
 // passes of up to VG vectors: scores (one thread per (v, position)), softmax
-// over the segment (one warp per v), P V (eight threads per (v, 4 dims),
+// over the segment (one warp per v), P V (eight threads per (v, 8 dims),
 // interleaved positions, fixed shuffle tree); the partial (o, max, sum) of the segment goes to
 // global memory.  After its items, a CTA adds its count to each KV head's
 // counter; the last arrival combines the segment partials of that head in
@@ -851,40 +851,43 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
             }
             consumer_sync();
 
-            // P V: eight threads per (v, 4 dims); thread g sums positions g, g + 8,
+            // P V: eight threads per (v, 8 dims); thread g sums positions g, g + 8,
             // ... in order (rows with distinct swizzle phases: no bank
             // conflicts), then a fixed shuffle tree over the eight
-            for (int k = tid; k < nv * (HD / 4) * 8; k += kConsumers) {
-                const int g = k & 7, e4 = (k >> 3) % (HD / 4), vl = k / (2 * HD);
+            for (int k = tid; k < nv * HD; k += kConsumers) {
+                const int g = k & 7, e8 = (k >> 3) % (HD / 8), vl = k / HD;
                 const int v = v0 + vl, m = v / G;
-                const int e = 4 * e4, bx = e >> 6, cc = (e & 63) >> 3, off = (e & 7) * 2;
-                float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+                const int e = 8 * e8, bx = e >> 6, cc = (e & 63) >> 3;
+                float acc[8];
+#pragma unroll
+                for (int x = 0; x < 8; ++x) acc[x] = 0.f;
                 for (int j = 0; j < n_u; ++j) {
                     const int n_t = min(kAttnChunk, pos0 + m + 1 - (t0 + j * kAttnChunk));  // <= 0: none
                     const float* pv = sc + vl * SP + j * kAttnChunk;
-                    const unsigned char* vb = smem + ((i + j) % S) * L::STAGE + 16384 + bx * 8192 + off;
-#pragma unroll 4
+                    const unsigned char* vb = smem + ((i + j) % S) * L::STAGE + 16384 + bx * 8192;
+#pragma unroll 2
                     for (int t = g; t < n_t; t += 8) {
-                        const uint2 va = *reinterpret_cast<const uint2*>(vb + t * 128 + ((cc ^ (t & 7)) << 4));
+                        const uint4 va = *reinterpret_cast<const uint4*>(vb + t * 128 + ((cc ^ (t & 7)) << 4));
                         const float pa = pv[t];
-                        const float2 x0 = f16x2(va.x), x1 = f16x2(va.y);
-                        a0 += pa * x0.x;
-                        a1 += pa * x0.y;
-                        a2 += pa * x1.x;
-                        a3 += pa * x1.y;
+                        const float2 x0 = f16x2(va.x), x1 = f16x2(va.y), x2 = f16x2(va.z), x3 = f16x2(va.w);
+                        acc[0] += pa * x0.x;
+                        acc[1] += pa * x0.y;
+                        acc[2] += pa * x1.x;
+                        acc[3] += pa * x1.y;
+                        acc[4] += pa * x2.x;
+                        acc[5] += pa * x2.y;
+                        acc[6] += pa * x3.x;
+                        acc[7] += pa * x3.y;
                     }
                 }
 #pragma unroll
-                for (int w = 1; w < 8; w <<= 1) {
-                    a0 += __shfl_xor_sync(0xffffffffu, a0, w);
-                    a1 += __shfl_xor_sync(0xffffffffu, a1, w);
-                    a2 += __shfl_xor_sync(0xffffffffu, a2, w);
-                    a3 += __shfl_xor_sync(0xffffffffu, a3, w);
-                }
-                if (g == 0) {
-                    float* o = part + (size_t)v * part_v + e;
-                    *reinterpret_cast<float2*>(o) = make_float2(a0, a1);
-                    *reinterpret_cast<float2*>(o + 2) = make_float2(a2, a3);
+                for (int w = 1; w < 8; w <<= 1)
+#pragma unroll
+                    for (int x = 0; x < 8; ++x) acc[x] += __shfl_xor_sync(0xffffffffu, acc[x], w);
+                if (g == 0) {  // partial rows are (HD + 2) floats: 8-byte aligned only
+                    float2* o = reinterpret_cast<float2*>(part + (size_t)v * part_v + e);
+#pragma unroll
+                    for (int x = 0; x < 4; ++x) o[x] = make_float2(acc[2 * x], acc[2 * x + 1]);
                 }
             }
             consumer_sync();  // scores / q of this pass are free
