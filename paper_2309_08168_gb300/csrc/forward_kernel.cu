@@ -212,6 +212,26 @@ __device__ __forceinline__ void prefetch_tmap(const void* tmap) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(tmap) : "memory");
 }
 
+// fp16 tensor-core MMA (attention: K / V are fp16) and 8x8 matrix loads
+__device__ __forceinline__ void mma_f16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                              uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 "
+        "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], const void* p) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(smem_u32(p)));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(smem_u32(p)));
+}
+
 // ---------------------------------------------------------------------------
 // projection op
 // ---------------------------------------------------------------------------
@@ -248,13 +268,18 @@ struct GemmSmem {
     static constexpr int XB = XR * ROWB;         // = 4 * XKB
     static constexpr int STAGE = WB + XB;
     static constexpr int RC = NT * 8;
-    static constexpr int VG = 16;  // attention: query vectors per pass over a staged segment
+    static constexpr int VG = 16;  // attention: query vectors per item (one MMA M / N tile)
     static constexpr int S = 4;  // ring depth (5 or 6 stages, where they fit, measured no faster)
     static constexpr int RED = S * STAGE;                // [64][RC] floats
     static constexpr int YS = RED + kTileRows * RC * 4;  // [64][16] floats
-    static constexpr int ATT = RED;                      // [VG][128] q, [VG][SEG] scores
+    // attention scratch: q hi / lo (fp16, rows padded by 16 bytes), scores
+    // (fp32), P hi / lo (fp16, padded rows)
+    static constexpr int QST = 128 + 8, PST = kAttnSegChunks * kAttnChunk + 8;  // halves per row
+    static constexpr int ATT = RED;
+    static constexpr int ATT_SC = ATT + 2 * VG * QST * 2;
+    static constexpr int ATT_P = ATT_SC + VG * kAttnSegChunks * kAttnChunk * 4;
     static constexpr int SCRATCH_GEMM = kTileRows * RC * 4 + kTileRows * 16 * 4;
-    static constexpr int SCRATCH_ATT = VG * 128 * 4 + VG * kAttnSegChunks * kAttnChunk * 4;
+    static constexpr int SCRATCH_ATT = ATT_P + 2 * VG * PST * 2 - ATT;
     static constexpr size_t BYTES =
         1024 + (size_t)RED + (SCRATCH_GEMM > SCRATCH_ATT ? SCRATCH_GEMM : SCRATCH_ATT);
 };
@@ -685,14 +710,16 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 // segment order (flash-decoding style split of the softmax).  Every reduction
 // has a fixed order that depends only on the row's own position, not on M.
 struct AttnRange {
-    int n_ch, n_seg, i_begin, i_end;  // chunks, segments per KV head; this CTA's items
+    int n_ch, n_seg, n_vg;  // chunks, segments per KV head, groups of 16 query vectors
+    int i_begin, i_end;     // this CTA's items (KV head, segment, vector group), group fastest
 };
 __device__ __forceinline__ AttnRange attn_range(const AttnArgs& a, int M, int pos0) {
     constexpr int S = kAttnSegChunks;
     AttnRange r;
     r.n_ch = (pos0 + M + kAttnChunk - 1) / kAttnChunk;  // chunks holding any visible position
     r.n_seg = (r.n_ch + S - 1) / S;
-    const long long I = (long long)a.n_kv_heads * r.n_seg, GR = gridDim.x;
+    r.n_vg = (a.n_heads / a.n_kv_heads * M + 15) / 16;
+    const long long I = (long long)a.n_kv_heads * r.n_seg * r.n_vg, GR = gridDim.x;
     r.i_begin = (int)((long long)blockIdx.x * I / GR);
     r.i_end = (int)((long long)(blockIdx.x + 1) * I / GR);
     return r;
@@ -709,7 +736,7 @@ __device__ int attn_produce(const AttnArgs& a, const AttnRange& ar, int pos0, un
     constexpr int S = L::S, SC = kAttnSegChunks;
     int i = 0;
     for (int it = ar.i_begin; it < ar.i_end; ++it) {
-        const int kvh = it / ar.n_seg, c0 = (it - kvh * ar.n_seg) * SC;
+        const int hs = it / ar.n_vg, kvh = hs / ar.n_seg, c0 = (hs - kvh * ar.n_seg) * SC;
         for (int c = c0; c < min(c0 + SC, ar.n_ch); ++c, ++i) {
             if (i < i_from) continue;
             if (i >= i_limit || (old_only && (c + 1) * kAttnChunk > pos0)) return i;
@@ -760,138 +787,138 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
         return attn_produce<R, HD>(a, ar, pos0, smem, pp, err, pre, 1 << 30, false) >= 0;
     }
 
-    float* qs = reinterpret_cast<float*>(smem + L::ATT);  // [VG][HD]
-    float* sc = qs + VG * HD;                              // [VG][SP] scores, then weights
+    constexpr int QST = L::QST, PST = L::PST;
+    __half* qh = reinterpret_cast<__half*>(smem + L::ATT);  // [VG][QST] q hi, then lo
+    __half* ql = qh + VG * QST;
+    float* sc = reinterpret_cast<float*>(smem + L::ATT_SC);  // [VG][SP] scores
+    __half* ph = reinterpret_cast<__half*>(smem + L::ATT_P);  // [VG][PST] weights hi, then lo
+    __half* pl = ph + VG * PST;
     __shared__ unsigned s_mask;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int g = lane >> 2, tg = lane & 3;
     const size_t part_v = HD + 2;  // floats per partial: o[HD], max, sum
-    int q_kvh = -1;
     bool ok = true;
     int i = 0;  // ring position within the op
 
     for (int it = ar.i_begin; it < ar.i_end; ++it) {
-        const int kvh = it / ar.n_seg, sg = it - kvh * ar.n_seg, t0 = sg * SP;
+        const int hs = it / ar.n_vg, vg = it - hs * ar.n_vg;
+        const int kvh = hs / ar.n_seg, sg = hs - kvh * ar.n_seg, t0 = sg * SP;
         const int n_u = min(SC, ar.n_ch - sg * SC);  // chunks of this segment
+        const int v0 = vg * VG, nv = min(VG, NV - v0);
         float* part = a.part + ((size_t)kvh * a.n_chunks + sg) * NV * part_v;
-        for (int v0 = 0; v0 < NV; v0 += VG) {
-            const int nv = min(VG, NV - v0);
-            if (kvh != q_kvh || NV > VG) {  // q of this pass (written by other CTAs: L2)
-                for (int k = tid; k < nv * HD; k += kConsumers) {
-                    const int v = v0 + k / HD, e = k % HD;
-                    const int m = v / G, gi = v - m * G;
-                    qs[k] = __ldcg(a.q + (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e);
-                }
-                q_kvh = kvh;
+        // q of this item's vectors as fp16 hi + lo (other CTAs wrote q: L2);
+        // the loads overlap the wait for K / V
+        for (int k = tid; k < VG * HD; k += kConsumers) {
+            const int vl = k / HD, e = k - vl * HD;
+            float x = 0.f;
+            if (vl < nv) {
+                const int v = v0 + vl, m = v / G, gi = v - m * G;
+                x = __ldcg(a.q + (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e);
             }
-            if (v0 == 0) {  // K / V of the segment (the q loads above overlap the wait)
-                for (int j = 0; j < n_u; ++j) {
-                    const int s = (i + j) % S;
-                    ok = mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err) && ok;
-                    pp.cphase ^= 1u << s;
-                }
-                if (ct && tid == 0 && it == ar.i_begin) ct[1] = globaltimer();
-            }
-            consumer_sync();
-            // scores: thread per (v, t); row m sees positions <= pos0 + m
-            for (int k = tid; k < nv * SP; k += kConsumers) {
-                const int vl = k / SP, t = k - vl * SP;
-                const int m = (v0 + vl) / G, j = t / kAttnChunk, tt = t - j * kAttnChunk;
-                float dot = -INFINITY;
-                if (j < n_u && t0 + t <= pos0 + m) {
-                    const unsigned char* ks = smem + ((i + j) % S) * L::STAGE;
-                    float d0 = 0.f, d1 = 0.f;
-                    const float4* q4 = reinterpret_cast<const float4*>(qs + vl * HD);
-                    const int sw = tt & 7;
-#pragma unroll
-                    for (int bx = 0; bx < HD / 64; ++bx) {
-#pragma unroll
-                        for (int cc = 0; cc < 8; ++cc) {
-                            const uint4 kv =
-                                *reinterpret_cast<const uint4*>(ks + bx * 8192 + tt * 128 + ((cc ^ sw) << 4));
-                            const float4 qa = q4[bx * 16 + cc * 2], qb = q4[bx * 16 + cc * 2 + 1];
-                            const float2 k0 = f16x2(kv.x), k1 = f16x2(kv.y), k2 = f16x2(kv.z), k3 = f16x2(kv.w);
-                            float& d = (cc & 1) ? d1 : d0;
-                            d += qa.x * k0.x + qa.y * k0.y;
-                            d += qa.z * k1.x + qa.w * k1.y;
-                            d += qb.x * k2.x + qb.y * k2.y;
-                            d += qb.z * k3.x + qb.w * k3.y;
-                        }
-                    }
-                    dot = (d0 + d1) * a.scale;
-                }
-                sc[k] = dot;
-            }
-            consumer_sync();
-
-            // softmax over the segment: warp per v, positions lane + 32 q
-            for (int vl = warp; vl < nv; vl += kConsumers / 32) {
-                const int v = v0 + vl, m = v / G;
-                float* o = part + (size_t)v * part_v;
-                float* sv = sc + vl * SP;
-                if (pos0 + m < t0) {  // nothing visible in this segment
-#pragma unroll
-                    for (int q = 0; q < SP / 32; ++q) sv[lane + 32 * q] = 0.f;
-                    if (lane == 0) { o[HD] = -INFINITY; o[HD + 1] = 0.f; }
-                    continue;
-                }
-                float mx = -INFINITY;
-#pragma unroll
-                for (int q = 0; q < SP / 32; ++q) mx = fmaxf(mx, sv[lane + 32 * q]);
-                mx = warp_max(mx);
-                float l = 0.f;
-#pragma unroll
-                for (int q = 0; q < SP / 32; ++q) {
-                    const float x = sv[lane + 32 * q];
-                    const float pq = x == -INFINITY ? 0.f : expf(x - mx);
-                    sv[lane + 32 * q] = pq;
-                    l += pq;
-                }
-                l = warp_sum(l);
-                if (lane == 0) { o[HD] = mx; o[HD + 1] = l; }
-            }
-            consumer_sync();
-
-            // P V: eight threads per (v, 8 dims); thread g sums positions g, g + 8,
-            // ... in order (rows with distinct swizzle phases: no bank
-            // conflicts), then a fixed shuffle tree over the eight
-            for (int k = tid; k < nv * HD; k += kConsumers) {
-                const int g = k & 7, e8 = (k >> 3) % (HD / 8), vl = k / HD;
-                const int v = v0 + vl, m = v / G;
-                const int e = 8 * e8, bx = e >> 6, cc = (e & 63) >> 3;
-                float acc[8];
-#pragma unroll
-                for (int x = 0; x < 8; ++x) acc[x] = 0.f;
-                for (int j = 0; j < n_u; ++j) {
-                    const int n_t = min(kAttnChunk, pos0 + m + 1 - (t0 + j * kAttnChunk));  // <= 0: none
-                    const float* pv = sc + vl * SP + j * kAttnChunk;
-                    const unsigned char* vb = smem + ((i + j) % S) * L::STAGE + 16384 + bx * 8192;
-#pragma unroll 2
-                    for (int t = g; t < n_t; t += 8) {
-                        const uint4 va = *reinterpret_cast<const uint4*>(vb + t * 128 + ((cc ^ (t & 7)) << 4));
-                        const float pa = pv[t];
-                        const float2 x0 = f16x2(va.x), x1 = f16x2(va.y), x2 = f16x2(va.z), x3 = f16x2(va.w);
-                        acc[0] += pa * x0.x;
-                        acc[1] += pa * x0.y;
-                        acc[2] += pa * x1.x;
-                        acc[3] += pa * x1.y;
-                        acc[4] += pa * x2.x;
-                        acc[5] += pa * x2.y;
-                        acc[6] += pa * x3.x;
-                        acc[7] += pa * x3.y;
-                    }
-                }
-#pragma unroll
-                for (int w = 1; w < 8; w <<= 1)
-#pragma unroll
-                    for (int x = 0; x < 8; ++x) acc[x] += __shfl_xor_sync(0xffffffffu, acc[x], w);
-                if (g == 0) {  // partial rows are (HD + 2) floats: 8-byte aligned only
-                    float2* o = reinterpret_cast<float2*>(part + (size_t)v * part_v + e);
-#pragma unroll
-                    for (int x = 0; x < 4; ++x) o[x] = make_float2(acc[2 * x], acc[2 * x + 1]);
-                }
-            }
-            consumer_sync();  // scores / q of this pass are free
+            const __half xh = __float2half_rn(x);
+            qh[vl * QST + e] = xh;
+            ql[vl * QST + e] = __float2half_rn(x - __half2float(xh));
         }
+        for (int j = 0; j < n_u; ++j) {
+            const int s = (i + j) % S;
+            ok = mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err) && ok;
+            pp.cphase ^= 1u << s;
+        }
+        if (ct && tid == 0 && it == ar.i_begin) ct[1] = globaltimer();
+        consumer_sync();
+
+        // scores S = K q^T on tensor cores: warp w takes positions 16w..16w+15
+        // (A = K rows, 128-byte swizzled), all 16 vectors (B = q hi, then lo)
+        {
+            const int p0 = warp * 16, j = p0 / kAttnChunk;
+            float c[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+            if (j < n_u) {
+                const unsigned char* kst = smem + ((i + j) % S) * L::STAGE;
+                const int t = (p0 % kAttnChunk) + (lane & 7) + 8 * ((lane >> 3) & 1);
+                const int qv = (lane & 7) + 8 * (lane >> 4), qk = ((lane >> 3) & 1) * 8;
+#pragma unroll
+                for (int ks = 0; ks < HD / 16; ++ks) {
+                    uint32_t af[4], bh[4], bl[4];
+                    const int chunk = 2 * (ks & 3) + (lane >> 4);
+                    ldsm_x4(af, kst + (ks >> 2) * 8192 + t * 128 + ((chunk ^ (t & 7)) << 4));
+                    ldsm_x4(bh, qh + qv * QST + ks * 16 + qk);
+                    ldsm_x4(bl, ql + qv * QST + ks * 16 + qk);
+                    mma_f16_16816(c[0], af[0], af[1], af[2], af[3], bh[0], bh[1]);
+                    mma_f16_16816(c[1], af[0], af[1], af[2], af[3], bh[2], bh[3]);
+                    mma_f16_16816(c[0], af[0], af[1], af[2], af[3], bl[0], bl[1]);
+                    mma_f16_16816(c[1], af[0], af[1], af[2], af[3], bl[2], bl[3]);
+                }
+            }
+            // C: rows = positions p0 + g (+8), columns = vectors 8 nt + 2 tg (+1)
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int x = 0; x < 4; ++x) {
+                    const int vl = nt * 8 + 2 * tg + (x & 1), pq = p0 + g + 8 * (x >> 1);
+                    const int m = (v0 + vl) / G;
+                    const bool vis = j < n_u && vl < nv && t0 + pq <= pos0 + m;
+                    sc[vl * SP + pq] = vis ? c[nt][x] * a.scale : -INFINITY;
+                }
+        }
+        consumer_sync();
+
+        // softmax over the segment: warp per vector; weights as fp16 hi + lo
+        for (int vl = warp; vl < nv; vl += kConsumers / 32) {
+            const int v = v0 + vl, m = v / G;
+            float* o = part + (size_t)v * part_v;
+            const float* sv = sc + vl * SP;
+            float mx = -INFINITY;
+#pragma unroll
+            for (int q = 0; q < SP / 32; ++q) mx = fmaxf(mx, sv[lane + 32 * q]);
+            mx = warp_max(mx);
+            float l = 0.f;
+#pragma unroll
+            for (int q = 0; q < SP / 32; ++q) {
+                const float x = sv[lane + 32 * q];
+                const float pq = x == -INFINITY ? 0.f : expf(x - mx);
+                const __half hh = __float2half_rn(pq);
+                ph[vl * PST + lane + 32 * q] = hh;
+                pl[vl * PST + lane + 32 * q] = __float2half_rn(pq - __half2float(hh));
+                l += pq;
+            }
+            l = warp_sum(l);
+            if (lane == 0) {
+                o[HD] = pos0 + m < t0 ? -INFINITY : mx;  // -inf: nothing visible in this segment
+                o[HD + 1] = l;
+            }
+        }
+        consumer_sync();
+
+        // O = P V on tensor cores: warp w takes dims 16w..16w+15 (B = V rows via
+        // transposed 8x8 loads), all 16 vectors (A = P hi, then lo); rows of
+        // vectors past nv hold stale weights and are not stored
+        if (warp * 16 < HD) {
+            float c[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+            const int d = warp * 16 + 8 * (lane >> 4), bx = d >> 6, cc = (d & 63) >> 3;
+            const int pv = (lane & 7) + 8 * ((lane >> 3) & 1), pk = (lane >> 4) * 8;
+            for (int ks = 0; ks < n_u * (kAttnChunk / 16); ++ks) {
+                uint32_t ah[4], al[4], bv[4];
+                const int p = ks * 16 + (lane & 7) + 8 * ((lane >> 3) & 1), j = p / kAttnChunk, tt = p % kAttnChunk;
+                ldsm_x4(ah, ph + pv * PST + ks * 16 + pk);
+                ldsm_x4(al, pl + pv * PST + ks * 16 + pk);
+                ldsm_x4_t(bv, smem + ((i + j) % S) * L::STAGE + 16384 + bx * 8192 + tt * 128 + ((cc ^ (tt & 7)) << 4));
+                mma_f16_16816(c[0], ah[0], ah[1], ah[2], ah[3], bv[0], bv[1]);
+                mma_f16_16816(c[1], ah[0], ah[1], ah[2], ah[3], bv[2], bv[3]);
+                mma_f16_16816(c[0], al[0], al[1], al[2], al[3], bv[0], bv[1]);
+                mma_f16_16816(c[1], al[0], al[1], al[2], al[3], bv[2], bv[3]);
+            }
+            // C: rows = vectors g (+8), columns = dims 16w + 8 nt + 2 tg (+1)
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int vl = g + 8 * h;
+                    if (vl < nv)
+                        *reinterpret_cast<float2*>(part + (size_t)(v0 + vl) * part_v + warp * 16 + nt * 8 + 2 * tg) =
+                            make_float2(c[nt][2 * h], c[nt][2 * h + 1]);
+                }
+        }
+        consumer_sync();  // q / scores / weights are free for the next item
         __syncwarp();
         if (lane == 0)
             for (int j = 0; j < n_u; ++j) mbar_arrive(pp.empty + (i + j) % S);  // the stages are free
@@ -907,16 +934,17 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
     // combines that head (all heads a CTA completes are combined in one pass)
     __threadfence();
     consumer_sync();
-    const int kv_lo = ar.i_begin / ar.n_seg, kv_hi = (ar.i_end - 1) / ar.n_seg;
+    const int per_kv = ar.n_seg * ar.n_vg;  // items of one KV head
+    const int kv_lo = ar.i_begin / per_kv, kv_hi = (ar.i_end - 1) / per_kv;
     for (int kb = kv_lo; kb <= kv_hi; kb += 32) {
         const int nk = min(32, kv_hi - kb + 1);
         if (warp == 0) {
             bool last = false;
             if (lane < nk) {
                 const int kvh = kb + lane;
-                const int cnt = min(ar.i_end, (kvh + 1) * ar.n_seg) - max(ar.i_begin, kvh * ar.n_seg);
+                const int cnt = min(ar.i_end, (kvh + 1) * per_kv) - max(ar.i_begin, kvh * per_kv);
                 const unsigned prev = atomicAdd(&a.counters[kvh], (unsigned)cnt);
-                last = prev + (unsigned)cnt == (unsigned)ar.n_seg;
+                last = prev + (unsigned)cnt == (unsigned)per_kv;
                 if (last) a.counters[kvh] = 0u;  // no other CTA touches it again in this op
             }
             const unsigned mask = __ballot_sync(0xffffffffu, last);
