@@ -74,11 +74,13 @@ __device__ bool grid_barrier(unsigned* bar, unsigned target, int* err) {
     __shared__ int s_ok;
     __syncthreads();
     if (threadIdx.x == 0) {
+        // the CTA's stores (ordered before this thread by the CTA barrier) are
+        // published by the fence; the arrival itself needs no reply
         __threadfence();
-        atomicAdd(bar, 1u);
+        asm volatile("red.relaxed.gpu.global.add.u32 [%0], 1;" ::"l"(bar) : "memory");
         int ok = 1;
         const unsigned long long t0 = globaltimer();
-        while (ld_acquire(bar) < target) {
+        while (ld_acquire(bar) < target) {  // acquire: later loads see the others' stores
             if (*(volatile int*)err) { ok = 0; break; }
             if (globaltimer() - t0 > kBarrierTimeoutNs) {
                 atomicCAS(err, 0, kDevErrTimeout);
@@ -87,7 +89,6 @@ __device__ bool grid_barrier(unsigned* bar, unsigned target, int* err) {
             }
             __nanosleep(32);
         }
-        __threadfence();
         s_ok = ok;
     }
     __syncthreads();
@@ -798,7 +799,8 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
     const int g = lane >> 2, tg = lane & 3;
     const size_t part_v = HD + 2;  // floats per partial: o[HD], max, sum
     bool ok = true;
-    int i = 0;  // ring position within the op
+    int i = 0;       // ring position within the op
+    int q_key = -1;  // (KV head, vector group) whose q is in shared memory
 
     for (int it = ar.i_begin; it < ar.i_end; ++it) {
         const int hs = it / ar.n_vg, vg = it - hs * ar.n_vg;
@@ -807,8 +809,10 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
         const int v0 = vg * VG, nv = min(VG, NV - v0);
         float* part = a.part + ((size_t)kvh * a.n_chunks + sg) * NV * part_v;
         // q of this item's vectors as fp16 hi + lo (other CTAs wrote q: L2);
-        // the loads overlap the wait for K / V
-        for (int k = tid; k < VG * HD; k += kConsumers) {
+        // the loads overlap the wait for K / V; consecutive items of one KV
+        // head and vector group reuse it
+        const int key = kvh * ar.n_vg + vg;
+        for (int k = key == q_key ? VG * HD : tid; k < VG * HD; k += kConsumers) {
             const int vl = k / HD, e = k - vl * HD;
             float x = 0.f;
             if (vl < nv) {
@@ -819,6 +823,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
             qh[vl * QST + e] = xh;
             ql[vl * QST + e] = __float2half_rn(x - __half2float(xh));
         }
+        q_key = key;
         for (int j = 0; j < n_u; ++j) {
             const int s = (i + j) % S;
             ok = mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err) && ok;
@@ -844,9 +849,11 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
                     ldsm_x4(bh, qh + qv * QST + ks * 16 + qk);
                     ldsm_x4(bl, ql + qv * QST + ks * 16 + qk);
                     mma_f16_16816(c[0], af[0], af[1], af[2], af[3], bh[0], bh[1]);
-                    mma_f16_16816(c[1], af[0], af[1], af[2], af[3], bh[2], bh[3]);
                     mma_f16_16816(c[0], af[0], af[1], af[2], af[3], bl[0], bl[1]);
-                    mma_f16_16816(c[1], af[0], af[1], af[2], af[3], bl[2], bl[3]);
+                    if (nv > 8) {  // vectors 8..15
+                        mma_f16_16816(c[1], af[0], af[1], af[2], af[3], bh[2], bh[3]);
+                        mma_f16_16816(c[1], af[0], af[1], af[2], af[3], bl[2], bl[3]);
+                    }
                 }
             }
             // C: rows = positions p0 + g (+8), columns = vectors 8 nt + 2 tg (+1)
