@@ -112,7 +112,7 @@ struct ssd_handle {
     bf16* ac_hi = nullptr;  // SwiGLU output planes [16][ffn]
     bf16* ac_lo = nullptr;
     int n_sms = 0;
-    unsigned* bar = nullptr;            // grid-barrier counter of the forward kernel
+    unsigned* bar = nullptr;            // grid-barrier counter of the forward kernel, then its sequence number
     unsigned long long* trace = nullptr;  // per-op timestamps (profiling hook, FwdParams::trace)
     int trace_op = -1;                    // op traced per unit and per CTA
     CUtensorMap* tmaps = nullptr;       // TMA descriptors (weights, input planes) in device memory
@@ -417,6 +417,7 @@ int forward(ssd_handle* h, int M, int src, const int* toks, int pos0, bool draft
     p.xn_lo = h->xn_lo;
     p.ss = h->ss;
     p.bar = h->bar;
+    p.seq = h->bar + 1;
     p.err = &h->st->err;
     p.trace = trace;
     p.trace_op = h->trace_op;
@@ -653,7 +654,8 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
         (rc = dalloc(h, &h->ac_hi, (size_t)2 * kMaxRows * F, &B)) ||
         (rc = dalloc(h, &h->logits, (size_t)kMaxRows * V, &B)) ||
         (rc = dalloc(h, &h->p_rows, (size_t)kMaxRows * V, &B)) ||
-        (rc = dalloc(h, &h->q_rows, (size_t)kMaxRows * V, &B)) || (rc = dalloc(h, &h->partial, part, &B)) ||
+        (rc = dalloc(h, &h->q_rows, (size_t)kMaxRows * V, &B)) ||
+        (rc = dalloc(h, &h->partial, 2 * part, &B)) ||  // tagged 64-bit words in the forward kernel
         (rc = dalloc(h, &h->counters, (size_t)tiles + c.n_kv_heads + 4, &B)) ||
         (rc = dalloc(h, &h->attn_part, (size_t)c.n_kv_heads * h->n_chunks * G * kMaxRows * (HD + 2), &B)) ||
         (rc = dalloc(h, &h->rope, (size_t)c.max_seq * (HD / 2), &B)) ||
@@ -691,6 +693,10 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
     }
     cudaError_t e = cudaMemsetAsync(h->counters, 0, ((size_t)tiles + c.n_kv_heads + 4) * sizeof(unsigned), h->stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(h->st, 0, sizeof(DecodeState), h->stream);
+    // barrier counter and forward sequence number; split-K slots hold no
+    // valid tag (a tag is never 0: GEMM ops have an op index >= 1)
+    if (e == cudaSuccess) e = cudaMemsetAsync(h->bar, 0, 4 * sizeof(unsigned), h->stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(h->partial, 0, 2 * part * sizeof(float), h->stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(h->kc, 0, h->kv_layer * L * sizeof(f16), h->stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(h->vc, 0, h->kv_layer * L * sizeof(f16), h->stream);
     if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);

@@ -19,15 +19,18 @@
 // activation rows as bf16 hi + lo planes on its N side (~16 mantissa bits).
 // Work unit = 64-row tile x 256-wide k chunk (32 KB of weights); each CTA
 // owns an equal contiguous range of units in tile-major order, streamed
-// through a 4-stage cp.async ring; a tile split over several CTAs is summed
-// in segment order by the CTA that finishes it last (arrival counter, no
-// waiting).  RMSNorm is folded in: the producer of the residual stream writes
-// the planes of h * g_next and per-64-column sums of h^2, the consumer scales
-// row m by rsqrt(mean(h^2) + eps) in its epilogue (W (h g r) = r W (h g)).
+// through a 4-stage TMA ring.  A tile split over several CTAs is summed in
+// segment order by the CTA holding its first chunks; the others store their
+// partials tagged with the op (value and tag in one 64-bit word), so they
+// neither fence nor signal, and the finaliser polls the words themselves.
+// RMSNorm is folded in: the producer of the residual stream writes the planes
+// of h * g_next and per-64-column sums of h^2, the consumer scales row m by
+// rsqrt(mean(h^2) + eps) in its epilogue (W (h g r) = r W (h g)).
 //
-// Attention: units = (KV head, absolute 64-position chunk); the partial
-// softmax of a row over a chunk depends only on the row and the chunk, and
-// the CTA that completes a head last combines its chunks in chunk order.
+// Attention: items = (KV head, absolute 128-position segment, group of 16
+// query vectors); the partial softmax of a row over a segment depends only on
+// the row and the segment, and the CTA that completes a head last combines
+// its segments in segment order.
 //
 // Coherence: L1 is not coherent across SMs within one launch, so every load of
 // data another CTA wrote during this launch goes through L2 (cp.async.cg,
@@ -95,19 +98,32 @@ __device__ bool grid_barrier(unsigned* bar, unsigned target, int* err) {
     return s_ok != 0;
 }
 
-// fire-and-forget release increment (publishes this thread's earlier stores)
-__device__ __forceinline__ void red_release_add(unsigned* p, unsigned v) {
-    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+// Split-K partials: a float and the tag of the op that wrote it (forward
+// sequence number << 10 | op index) in one 64-bit word, written and read as
+// single 64-bit accesses.
+__device__ __forceinline__ unsigned long long tagged(unsigned tag, float v) {
+    return ((unsigned long long)tag << 32) | __float_as_uint(v);
 }
-
-// Bounded wait until *c >= target (acquire); false (timeout recorded) after
-// kBarrierTimeoutNs or when another CTA already recorded an error.
-__device__ bool wait_count(const unsigned* c, unsigned target, int* err) {
-    if (ld_acquire(c) >= target) return true;
+__device__ __forceinline__ unsigned tag_of(unsigned long long w) { return (unsigned)(w >> 32); }
+__device__ __forceinline__ float value_of(unsigned long long w) { return __uint_as_float((unsigned)w); }
+__device__ __forceinline__ void st_relaxed_u64(unsigned long long* p, unsigned long long v) {
+    asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
+    unsigned long long v;
+    asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+// Bounded wait until the word at p carries `tag` (w: the word read); false
+// (timeout recorded) after kBarrierTimeoutNs or when another CTA already
+// recorded an error.  Kept out of line: inlined into the projection op, this
+// cold loop measurably slowed its MMA loop.
+__device__ __noinline__ bool wait_tag(const unsigned long long* p, unsigned tag, unsigned long long& w, int* err) {
     const unsigned long long t0 = globaltimer();
     for (;;) {
         __nanosleep(32);
-        if (ld_acquire(c) >= target) return true;
+        w = ld_relaxed_u64(p);
+        if (tag_of(w) == tag) return true;
         if (*(volatile int*)err) return false;
         if (globaltimer() - t0 > kBarrierTimeoutNs) {
             atomicCAS(err, 0, kDevErrTimeout);
@@ -413,7 +429,7 @@ __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, P
 // CTA's op stamps (FwdParams::trace) - profiling aids.
 template <int R>
 __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefetched, unsigned char* smem,
-                        float* r_s, Pipe& pp, const FwdOp* nx, int* err, unsigned long long* ut,
+                        float* r_s, Pipe& pp, unsigned tag, int* err, unsigned long long* ut,
                         unsigned long long* ct) {
     using L = GemmSmem<R>;
     constexpr int NT = L::NT, RC = L::RC;
@@ -550,6 +566,28 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
         consumer_sync();
+
+        // split-K: the CTA holding the tile's first chunks (its segment ends
+        // last, at the end of that CTA's range) finalises; the others store
+        // their partial (hi + lo plane columns summed) and move on.  Each value
+        // travels with the op's tag in one 64-bit word, so the finaliser needs
+        // no flag and no fence: it reads each word until the tag is this op's.
+        // The sum is in segment order.
+        const long long u_first = (long long)tile * a.n_chunks;
+        const int seg0 = unit_owner(u_first, U, G);
+        const int nseg = unit_owner(u_first + a.n_chunks - 1, U, G) - seg0 + 1;
+        constexpr size_t kSlot = (size_t)kMaxRows * kTileRows;
+        unsigned long long* slots =
+            reinterpret_cast<unsigned long long*>(a.partial) + (size_t)tile * a.n_chunks * kSlot;
+        if (nseg > 1 && b != seg0) {
+            unsigned long long* mine = slots + (size_t)(b - seg0) * kSlot;
+            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+                const int m = idx / kTileRows, r = idx - m * kTileRows;
+                st_relaxed_u64(mine + m * kTileRows + r, tagged(tag, red[r * RC + m] + red[r * RC + R + m]));
+            }
+            consumer_sync();  // red is free for the next segment
+            continue;
+        }
         for (int idx = threadIdx.x; idx < kTileRows * M; idx += kGemmThreads) {
             const int m = idx / kTileRows, r = idx - m * kTileRows;
             ys[r * 16 + m] = red[r * RC + m] + red[r * RC + R + m];
@@ -557,7 +595,7 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         consumer_sync();
 
         // RESID: this tile's residual h (written by earlier ops: L2), loaded
-        // before the split-K exchange so its latency overlaps it
+        // before waiting for the other segments so its latency overlaps it
         constexpr int HJ = kMaxRows * kTileRows / kGemmThreads;
         float hpre[HJ], gpre[HJ];
         if (epi == EPI_RESID) {
@@ -571,37 +609,25 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
             }
         }
 
-        // split-K: the CTA holding the tile's first chunks (its segment ends
-        // last, at the end of that CTA's range) finalises; the others publish
-        // their partial and move on.  The sum is in segment order.
-        const long long u_first = (long long)tile * a.n_chunks;
-        const int seg0 = unit_owner(u_first, U, G);
-        const int nseg = unit_owner(u_first + a.n_chunks - 1, U, G) - seg0 + 1;
         if (nseg > 1) {
-            float* slots = a.partial + (size_t)tile * a.n_chunks * kMaxRows * kTileRows;
-            if (b != seg0) {
-                float* mine = slots + (size_t)(b - seg0) * kMaxRows * kTileRows;
-                for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
-                    const int m = idx / kTileRows, r = idx - m * kTileRows;
-                    mine[m * kTileRows + r] = ys[r * 16 + m];
-                }
-                __threadfence();
-                consumer_sync();
-                if (threadIdx.x == 0) red_release_add(&a.counters[tile], 1u);
-                continue;
-            }
             // the other segments come from later CTAs, which never wait on this one
-            if (threadIdx.x == 0) {
-                if (!wait_count(&a.counters[tile], (unsigned)(nseg - 1), err)) ok = false;
-                a.counters[tile] = 0u;  // every other segment has been counted
-            }
-            consumer_sync();
             for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
                 const int m = idx / kTileRows, r = idx - m * kTileRows;
-                const float* p = slots + m * kTileRows + r;
+                const unsigned long long* p = slots + m * kTileRows + r;
                 float sum = ys[r * 16 + m];
-#pragma unroll 4
-                for (int sg = 1; sg < nseg; ++sg) sum += __ldcg(p + (size_t)sg * kMaxRows * kTileRows);
+                for (int sg0 = 1; sg0 < nseg; sg0 += 4) {
+                    unsigned long long w[4];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        if (sg0 + j < nseg) w[j] = ld_relaxed_u64(p + (size_t)(sg0 + j) * kSlot);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        if (sg0 + j < nseg) {
+                            if (tag_of(w[j]) != tag && !wait_tag(p + (size_t)(sg0 + j) * kSlot, tag, w[j], err))
+                                ok = false;
+                            sum += value_of(w[j]);
+                        }
+                }
                 ys[r * 16 + m] = sum;
             }
             consumer_sync();
@@ -1065,6 +1091,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     __shared__ float r_s[kMaxRows];
     __shared__ int s_pos0, s_fail;
+    __shared__ unsigned s_seq;
     constexpr int S = GemmSmem<R>::S;
     __shared__ __align__(8) uint64_t full[S];   // TMA completion per stage
     __shared__ __align__(8) uint64_t empty[S];  // stage released by the 8 consumer warps
@@ -1078,6 +1105,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         else pos0 = p.st->len;
         s_pos0 = pos0;
         s_fail = 0;
+        s_seq = *(volatile unsigned*)p.seq;  // this forward's number (advanced by CTA 0 below)
         for (int st = 0; st < S; ++st) {
             mbar_init(full + st, 1);
             mbar_init(empty + st, kConsumers / 32);
@@ -1109,7 +1137,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
             nx = s_op + ((o + 1) & 1);
         }
         if (is_gemm(type)) {
-            ok = gemm_op<R>(op.g, epi_of(type), p.M, pos0, prefetched, smem, r_s, pp, nx, p.err,
+            ok = gemm_op<R>(op.g, epi_of(type), p.M, pos0, prefetched, smem, r_s, pp, (s_seq << 10) | (unsigned)o, p.err,
                             (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr, ct);
         } else {
             if (type == OP_EMBED) embed_op(p, pos0);
@@ -1138,6 +1166,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
                 drain_before_exit();
                 return;
             }
+            // every CTA has read the sequence number before the first barrier
+            if (target == gridDim.x && blockIdx.x == 0 && threadIdx.x == 0) *p.seq = s_seq + 1u;
         }
         if (ct && threadIdx.x == 0) ct[5] = globaltimer();
         if (p.trace && blockIdx.x == 0 && threadIdx.x == 0) p.trace[o + 1] = globaltimer();

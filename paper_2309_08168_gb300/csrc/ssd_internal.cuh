@@ -55,8 +55,9 @@ struct GemmArgs {
     int n_tiles;         // row tiles
     const float* x;      // activations [M][K] fp32 (split into bf16 hi + lo in the kernel)
     int M;               // activation rows (1..16)
-    float* partial;      // [ksplit][M][n_tiles*64] split-K partial sums
-    unsigned* counters;  // [n_tiles] arrival counters (left at zero)
+    float* partial;      // split-K partials: gemm.cu [ksplit][M][n_tiles*64] floats; forward
+                         // kernel [n_tiles][n_chunks][16][64] tagged 64-bit words
+    unsigned* counters;  // [n_tiles] arrival counters of gemm.cu (left at zero)
     // epilogue operands
     float* out_f32;      // EPI_LOGITS: [M][ldo]; EPI_RESID: residual h [M][ldo]
     int ldo;
@@ -143,6 +144,7 @@ struct FwdParams {
     bf16* xn_lo;
     float* ss;            // per-64-column sums of h^2 [16][d/64]
     unsigned* bar;        // grid-barrier counter, zero at launch
+    unsigned* seq;        // forward sequence number (tags split-K partials; +1 per launch)
     int* err;             // device error code
     // Profiling hook: nullptr, or globaltimer stamps: [0, n_ops] start, end of
     // op o (CTA 0); [1024, 1280) CTA 0's first 64 units of op trace_op (producer
