@@ -175,9 +175,12 @@ int ssd_debug_time_forward(ssd_handle* h, int draft, int rows, int gemm_only, in
  * embedding, 1 q/k/v projection, 2 attention, 3 output or down projection,
  * 4 gate/up projection, 5 lm_head.  max_ops >= 2 + 5 * n_layers is always
  * enough.  detail_op: index of one op to trace in detail (-1: none).
- * unit_trace (may be NULL): 256 globaltimer stamps (ns) of CTA 0's first 64
- * work units of detail_op when it is a projection, 4 per unit: producer
+ * unit_trace (may be NULL): 256 globaltimer stamps (ns) of CTA 0 for
+ * detail_op.  A projection: its first 64 work units, 4 per unit: producer
  * issue, consumer data ready, MMA done, segment flush done (0 if none).
+ * Attention: its first 31 items, 8 per item: item start, q loaded, K / V
+ * ready, after the CTA barrier, scores done, softmax done, P V done, 0; then
+ * [248] partials published, [249] head counts added, [250] combine done.
  * cta_trace (may be NULL): 8 stamps per CTA of the forward kernel for
  * detail_op: op start, first data ready, last MMA done, work done, grid
  * barrier arrive, barrier release, number of work units, 0; max_ctas >= the

@@ -800,7 +800,7 @@ __device__ int attn_prefetch(const AttnArgs& a, int M, int pos0, unsigned char* 
 // producer already filled before the grid barrier (attn_prefetch).
 template <int R, int HD>
 __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem, Pipe& pp, int* err,
-                        unsigned long long* ct, int pre) {
+                        unsigned long long* ct, int pre, unsigned long long* ut) {
     using L = GemmSmem<R>;
     constexpr int S = L::S, VG = L::VG, SC = kAttnSegChunks, SP = SC * kAttnChunk;  // positions per segment
     static_assert(SC <= S, "a segment's chunks are held in the ring at once");
@@ -828,7 +828,12 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
     int i = 0;       // ring position within the op
     int q_key = -1;  // (KV head, vector group) whose q is in shared memory
 
+    // profiling aid: ut (CTA 0 of a traced forward) gets per-item phase stamps
+    auto stamp = [&](int it, int k) {
+        if (ut && tid == 0 && it - ar.i_begin < 31) ut[(it - ar.i_begin) * 8 + k] = globaltimer();
+    };
     for (int it = ar.i_begin; it < ar.i_end; ++it) {
+        stamp(it, 0);
         const int hs = it / ar.n_vg, vg = it - hs * ar.n_vg;
         const int kvh = hs / ar.n_seg, sg = hs - kvh * ar.n_seg, t0 = sg * SP;
         const int n_u = min(SC, ar.n_ch - sg * SC);  // chunks of this segment
@@ -850,13 +855,16 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
             ql[vl * QST + e] = __float2half_rn(x - __half2float(xh));
         }
         q_key = key;
+        stamp(it, 1);
         for (int j = 0; j < n_u; ++j) {
             const int s = (i + j) % S;
             ok = mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err) && ok;
             pp.cphase ^= 1u << s;
         }
         if (ct && tid == 0 && it == ar.i_begin) ct[1] = globaltimer();
+        stamp(it, 2);
         consumer_sync();
+        stamp(it, 3);
 
         // scores S = K q^T on tensor cores: warp w takes positions 16w..16w+15
         // (A = K rows, 128-byte swizzled), all 16 vectors (B = q hi, then lo)
@@ -894,6 +902,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
                 }
         }
         consumer_sync();
+        stamp(it, 4);
 
         // softmax over the segment: warp per vector; weights as fp16 hi + lo
         for (int vl = warp; vl < nv; vl += kConsumers / 32) {
@@ -921,6 +930,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
             }
         }
         consumer_sync();
+        stamp(it, 5);
 
         // O = P V on tensor cores: warp w takes dims 16w..16w+15 (B = V rows via
         // transposed 8x8 loads), all 16 vectors (A = P hi, then lo); rows of
@@ -952,6 +962,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
                 }
         }
         consumer_sync();  // q / scores / weights are free for the next item
+        stamp(it, 6);
         __syncwarp();
         if (lane == 0)
             for (int j = 0; j < n_u; ++j) mbar_arrive(pp.empty + (i + j) % S);  // the stages are free
@@ -967,6 +978,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
     // combines that head (all heads a CTA completes are combined in one pass)
     __threadfence();
     consumer_sync();
+    if (ut && tid == 0) ut[248] = globaltimer();
     const int per_kv = ar.n_seg * ar.n_vg;  // items of one KV head
     const int kv_lo = ar.i_begin / per_kv, kv_hi = (ar.i_end - 1) / per_kv;
     for (int kb = kv_lo; kb <= kv_hi; kb += 32) {
@@ -984,6 +996,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
             if (lane == 0) s_mask = mask;
         }
         consumer_sync();
+        if (ut && tid == 0) ut[249] = globaltimer();
         const int n_last = __popc(s_mask);
         if (n_last) {
             __threadfence();
@@ -1029,6 +1042,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
             }
         }
         consumer_sync();
+        if (ut && tid == 0) ut[250] = globaltimer();
     }
     return ok;
 }
@@ -1130,28 +1144,44 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         bool ok = true;
         unsigned long long* ct = (p.trace && o == p.trace_op) ? p.trace + kTraceCtas + blockIdx.x * 8 : nullptr;
         if (ct && threadIdx.x == 0) ct[0] = globaltimer();
-        // the next op's arguments (its slot held op o-1, finished by every thread)
-        const FwdOp* nx = nullptr;
-        if (o + 1 < p.n_ops) {
-            copy_op(p.ops + o + 1, s_op + ((o + 1) & 1));  // (all threads, includes a barrier)
-            nx = s_op + ((o + 1) & 1);
-        }
+        // the next op's arguments: the producer warp copies them (16 bytes a
+        // lane, asynchronously) into their slot, which held op o-1, while op
+        // o runs; the producer uses them as soon as it has issued op o
+        constexpr int kOpChunks = (int)(sizeof(FwdOp) / 16);
+        static_assert(sizeof(FwdOp) % 16 == 0 && kOpChunks <= 32, "an op is copied in 16-byte pieces by one warp");
+        const bool has_nx = o + 1 < p.n_ops;
+        const int plane = (int)threadIdx.x - kConsumers;  // lane in the producer warp
+        if (has_nx && plane >= 0 && plane < kOpChunks)
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                             smem_u32(reinterpret_cast<unsigned char*>(s_op + ((o + 1) & 1)) + 16 * plane)),
+                         "l"(reinterpret_cast<const unsigned char*>(p.ops + o + 1) + 16 * plane)
+                         : "memory");
         if (is_gemm(type)) {
             ok = gemm_op<R>(op.g, epi_of(type), p.M, pos0, prefetched, smem, r_s, pp, (s_seq << 10) | (unsigned)o, p.err,
                             (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr, ct);
         } else {
             if (type == OP_EMBED) embed_op(p, pos0);
-            else ok = attn_op<R, HD>(op.at, p.M, pos0, smem, pp, p.err, ct, attn_pre);
+            else ok = attn_op<R, HD>(op.at, p.M, pos0, smem, pp, p.err, ct, attn_pre,
+                                     (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr);
         }
         if (ct && threadIdx.x == 0) ct[3] = globaltimer();
+        // next op: visible to the producer warp now, to every thread after
+        // the CTA barrier below
+        if (plane >= 0) {
+            asm volatile("cp.async.wait_all;" ::: "memory");
+            __syncwarp();
+        }
+        const FwdOp* nx = has_nx ? s_op + ((o + 1) & 1) : nullptr;
         prefetched = false;
         attn_pre = 0;
-        if (nx && ok && is_gemm(nx->type)) {
-            ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err);
-            prefetched = true;
-        } else if (nx && ok && nx->type == OP_ATTN) {
-            attn_pre = attn_prefetch<R, HD>(nx->at, p.M, pos0, smem, pp, p.err);
-            ok = attn_pre >= 0;
+        if (plane == 0 && nx && ok) {
+            if (is_gemm(nx->type)) {
+                ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err);
+                prefetched = true;
+            } else if (nx->type == OP_ATTN) {
+                attn_pre = attn_prefetch<R, HD>(nx->at, p.M, pos0, smem, pp, p.err);
+                ok = attn_pre >= 0;
+            }
         }
         if (!ok) s_fail = 1;
         __syncthreads();

@@ -122,7 +122,7 @@ struct AttnArgs {
 enum OpType { OP_EMBED = 0, OP_QKV = 1, OP_ATTN = 2, OP_RESID = 3, OP_SWIGLU = 4, OP_LOGITS = 5 };
 constexpr int kDevErrTimeout = 1;  // DecodeState::err: a grid barrier or a TMA wait gave up
 
-struct FwdOp {
+struct alignas(16) FwdOp {  // (copied in 16-byte pieces)
     int type;
     GemmArgs g;   // projection ops
     AttnArgs at;  // attention op
