@@ -15,6 +15,11 @@ Parity status per function (pins are in tests/test_oracle_*.py):
   orc_spec_verify                     pinned: output law integrates to p
   orc_nucleus_probs / orc_sample      pinned: hand-worked golden cases
   orc_philox4x32_10                   pinned: published known-answer vectors
+  orc_exit_update (Eqs. 2-4)          pinned: closed forms of the gamma / AR
+                                      recurrences (constant and alternating AR_e)
+  orc_generate_ex (draft exit,        pinned: gamma = 0 reproduces no exit,
+    Algs. 3 / 4)                      gamma > 1 drafts once per round, lossless
+                                      invariant SSD == AR with exit
 """
 from __future__ import annotations
 
@@ -55,6 +60,14 @@ class OrcWeights(ctypes.Structure):
                [(n, _PP) for n in ("wq", "wk", "wv", "wo", "attn_norm", "w_gate", "w_up", "w_down", "mlp_norm")]
 
 
+class OrcExit(ctypes.Structure):
+    _fields_ = [("on", ctypes.c_int)] + [(n, ctypes.c_double) for n in ("gamma0", "alpha", "eps", "beta1", "beta2")]
+
+
+class OrcExitState(ctypes.Structure):
+    _fields_ = [("gamma", ctypes.c_double), ("ar", ctypes.c_double), ("e", ctypes.c_int)]
+
+
 class OrcStats(ctypes.Structure):
     _fields_ = [("rounds", ctypes.c_int), ("drafted", ctypes.c_int), ("accepted", ctypes.c_int),
                 ("emitted", ctypes.c_int), ("hist", ctypes.c_int * 33)]
@@ -81,6 +94,11 @@ def lib():
                                    ctypes.c_uint64, ctypes.c_double, ctypes.c_double, _P, _P,
                                    ctypes.POINTER(OrcStats), _P, _P]
         L.orc_generate.restype = ctypes.c_int
+        L.orc_generate_ex.argtypes = L.orc_generate.argtypes + [ctypes.POINTER(OrcExit), _P, _P]
+        L.orc_generate_ex.restype = ctypes.c_int
+        L.orc_exit_update.argtypes = [ctypes.POINTER(OrcExitState), ctypes.POINTER(OrcExit), ctypes.c_double]
+        L.orc_softmax_max.argtypes = [_P, ctypes.c_int]
+        L.orc_softmax_max.restype = ctypes.c_double
         L.orc_rmsnorm.argtypes = [_P, _P, ctypes.c_int, ctypes.c_double, _P]
         L.orc_rope.argtypes = [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_double]
         L.orc_philox4x32_10.argtypes = [_P, _P, _P]
@@ -178,7 +196,11 @@ class Oracle:
             self.n_layers, self.max_seq, self.w.n_kv_heads * self.w.head_dim)
 
     def generate(self, prompt, n_new: int, K: int, mode: int = 0, seed: int = 0,
-                 temperature: float = 1.0, top_p: float = 1.0, mask=None, want_logits=False):
+                 temperature: float = 1.0, top_p: float = 1.0, mask=None, want_logits=False,
+                 draft_exit=None):
+        """draft_exit: None, or (gamma0, alpha, eps, beta1, beta2) of the
+        adaptive draft exit; stats then also hold every round's draft count
+        ("keff") and gamma after its update ("gamma")."""
         p = np.ascontiguousarray(prompt, dtype=np.int32)
         m = self._mask(mask)
         out = np.zeros(n_new, dtype=np.int32)
@@ -187,13 +209,18 @@ class Oracle:
         if want_logits:
             dl = np.zeros((max(K, 1), self.w.vocab), dtype=np.float64)
             vl = np.zeros((K + 1, self.w.vocab), dtype=np.float64)
-        rc = lib().orc_generate(self.h, _ptr(p), p.size, n_new, K, mode, seed, temperature, top_p,
-                                None if m is None else _ptr(m), _ptr(out), ctypes.byref(st),
-                                None if dl is None else _ptr(dl), None if vl is None else _ptr(vl))
+        ex = OrcExit(0, 0.0, 0.0, 0.0, 0.0, 0.0) if draft_exit is None else OrcExit(1, *map(float, draft_exit))
+        keff = np.zeros(max(n_new, 1), dtype=np.int32)
+        gam = np.zeros(max(n_new, 1), dtype=np.float64)
+        rc = lib().orc_generate_ex(self.h, _ptr(p), p.size, n_new, K, mode, seed, temperature, top_p,
+                                   None if m is None else _ptr(m), _ptr(out), ctypes.byref(st),
+                                   None if dl is None else _ptr(dl), None if vl is None else _ptr(vl),
+                                   ctypes.byref(ex), _ptr(keff), _ptr(gam))
         if rc:
             raise ValueError(f"orc_generate failed ({rc})")
         stats = {"rounds": st.rounds, "drafted": st.drafted, "accepted": st.accepted,
-                 "emitted": st.emitted, "hist": list(st.hist)}
+                 "emitted": st.emitted, "hist": list(st.hist),
+                 "keff": keff[:st.rounds].tolist(), "gamma": gam[:st.rounds].tolist()}
         if want_logits:
             return out, stats, dl, vl
         return out, stats
@@ -267,3 +294,16 @@ def spec_verify_batch(p_rows, q_rows, drafts, r, ures):
     out = np.empty((T, 2), dtype=np.int32)
     lib().orc_spec_verify_batch(_ptr(p), _ptr(q), Kd, p.shape[1], T, _ptr(d), _ptr(rr), _ptr(uu), _ptr(out))
     return out[:, 0], out[:, 1]
+
+
+def exit_update(state, params, ar_e):
+    """One application of Eqs. 2-4: state = (gamma, ar, e), params = (gamma0,
+    alpha, eps, beta1, beta2); returns the new state."""
+    st = OrcExitState(*state)
+    lib().orc_exit_update(ctypes.byref(st), ctypes.byref(OrcExit(1, *map(float, params))), float(ar_e))
+    return st.gamma, st.ar, st.e
+
+
+def softmax_max(logits):
+    x = np.ascontiguousarray(logits, dtype=np.float64)
+    return lib().orc_softmax_max(_ptr(x), x.size)

@@ -48,6 +48,15 @@
  *   - RoPE pairs element i with element i + head_dim/2 (rotate-half form),
  *     frequency theta^(-2i/head_dim); GQA query head h reads KV head
  *     floor(h * n_kv_heads / n_heads).
+ *   - Adaptive draft exit (Sec. 3.4, Eqs. 2-4, Algorithms 3 / 4 of App. G):
+ *     the draft whose confidence falls below gamma is kept as the round's
+ *     last draft (the algorithms choose x_{j+1} before the test); confidence
+ *     is the largest probability of the distribution the draft was chosen
+ *     from (softmax of the draft logits in greedy mode, the temperature /
+ *     nucleus distribution q_j in sampling mode); AR_e = accepted / drafted
+ *     of round e; gamma and AR are updated after every verification that
+ *     had drafts, with beta1 = 0 at the first update; gamma starts at
+ *     gamma0 for every generation.
  */
 #include <math.h>
 #include <stdint.h>
@@ -485,6 +494,42 @@ void orc_spec_verify_batch(const double* p, const double* q, int Kd, int V, int 
 }
 
 /* ------------------------------------------------------------------------ */
+/* adaptive draft exit (Sec. 3.4, Eqs. 2-4)                                  */
+/* ------------------------------------------------------------------------ */
+
+typedef struct {
+    int on; /* 0: Algorithm 2 / 4 without exit */
+    double gamma0, alpha, eps, beta1, beta2;
+} orc_exit_params;
+
+typedef struct {
+    double gamma, ar;
+    int e; /* updates done */
+} orc_exit_state;
+
+/* After the verification of round e, with AR_e = accepted / drafted:
+ *   AR <- beta1 AR + (1 - beta1) AR_e            (beta1 = 0 at e = 1)
+ *   gamma~ = gamma + eps if AR <= alpha, else gamma - eps
+ *   gamma <- beta2 gamma + (1 - beta2) gamma~ */
+void orc_exit_update(orc_exit_state* s, const orc_exit_params* p, double ar_e) {
+    double b1 = s->e == 0 ? 0.0 : p->beta1;
+    s->ar = b1 * s->ar + (1.0 - b1) * ar_e;
+    double gt = s->ar <= p->alpha ? s->gamma + p->eps : s->gamma - p->eps;
+    s->gamma = p->beta2 * s->gamma + (1.0 - p->beta2) * gt;
+    s->e++;
+}
+
+/* Largest probability of softmax(logits): 1 / sum_x exp(l_x - max l). */
+double orc_softmax_max(const double* logits, int V) {
+    double mx = logits[0];
+    for (int i = 1; i < V; ++i)
+        if (logits[i] > mx) mx = logits[i];
+    double s = 0.0;
+    for (int i = 0; i < V; ++i) s += exp(logits[i] - mx);
+    return 1.0 / s;
+}
+
+/* ------------------------------------------------------------------------ */
 /* decoding loops: Algorithm 1 (K = 0), Algorithm 2 / Algorithm 4 (K > 0)    */
 /* ------------------------------------------------------------------------ */
 
@@ -498,11 +543,15 @@ int orc_prefill(orc_model* m, const int* prompt, int n_prompt) {
 /* mode 0 greedy, 1 sampling.  mask: 2*n_layers bytes (the draft's z).
  * out_tokens: n_new emitted tokens.  Optional: draft_logits_out /
  * verify_logits_out receive the first round's K_eff x V draft logits and
- * (K_eff+1) x V verification logits.  Returns 0 or a negative error. */
-int orc_generate(orc_model* m, const int* prompt, int n_prompt, int n_new, int K, int mode,
-                 uint64_t seed, double temperature, double top_p, const uint8_t* mask,
-                 int* out_tokens, orc_stats* stats, double* draft_logits_out,
-                 double* verify_logits_out) {
+ * (K_eff+1) x V verification logits; ex (NULL or ex->on == 0: no exit) turns
+ * on the adaptive draft exit, and then keff_out / gamma_out (n_new entries
+ * each, may be NULL) receive every round's draft count and its gamma after
+ * the round's update.  Returns 0 or a negative error. */
+int orc_generate_ex(orc_model* m, const int* prompt, int n_prompt, int n_new, int K, int mode,
+                    uint64_t seed, double temperature, double top_p, const uint8_t* mask,
+                    int* out_tokens, orc_stats* stats, double* draft_logits_out,
+                    double* verify_logits_out, const orc_exit_params* ex, int* keff_out,
+                    double* gamma_out) {
     const orc_config* c = &m->c;
     int V = c->vocab;
     if (n_new < 0 || K < 0 || K > 32 || n_prompt < 1) return -1;
@@ -519,6 +568,8 @@ int orc_generate(orc_model* m, const int* prompt, int n_prompt, int n_new, int K
     int x_last = prompt[n_prompt - 1];
     int emitted = 0;
     int first_round = 1;
+    const int exit_on = ex && ex->on;
+    orc_exit_state es = {exit_on ? ex->gamma0 : 0.0, 0.0, 0};
     while (emitted < n_new) {
         int remaining = n_new - emitted;
         int Kd = K < remaining - 1 ? K : remaining - 1;
@@ -528,12 +579,19 @@ int orc_generate(orc_model* m, const int* prompt, int n_prompt, int n_new, int K
             orc_forward(m, tin, len + j - 1, mask, logits);
             if (first_round && draft_logits_out)
                 memcpy(draft_logits_out + (size_t)(j - 1) * V, logits, sizeof(double) * V);
+            double conf;
             if (mode == 0) {
                 drafts[j - 1] = orc_argmax(logits, V);
+                conf = exit_on ? orc_softmax_max(logits, V) : 1.0;
             } else {
                 double* qj = Q + (size_t)(j - 1) * V;
                 orc_nucleus_probs(logits, V, temperature, top_p, qj);
                 drafts[j - 1] = orc_sample(qj, V, orc_uniform(seed, len + j, 0));
+                conf = exit_on ? qj[orc_argmax(qj, V)] : 1.0;
+            }
+            if (exit_on && conf < es.gamma) { /* draft exit: d_j is the last draft */
+                Kd = j;
+                break;
             }
         }
         /* verification stage: the full model on [x_last, d_1..d_Kd] */
@@ -564,6 +622,9 @@ int orc_generate(orc_model* m, const int* prompt, int n_prompt, int n_new, int K
         }
         for (int j = 0; j < n; ++j) out_tokens[emitted++] = drafts[j];
         out_tokens[emitted++] = y;
+        if (exit_on && Kd > 0) orc_exit_update(&es, ex, (double)n / Kd);
+        if (keff_out) keff_out[st.rounds] = Kd;
+        if (gamma_out) gamma_out[st.rounds] = es.gamma;
         st.rounds++;
         st.drafted += Kd;
         st.accepted += n;
@@ -576,4 +637,13 @@ int orc_generate(orc_model* m, const int* prompt, int n_prompt, int n_new, int K
     if (stats) *stats = st;
     free(logits); free(P); free(Q);
     return 0;
+}
+
+/* Algorithm 1 / 2 / 4 without draft exit. */
+int orc_generate(orc_model* m, const int* prompt, int n_prompt, int n_new, int K, int mode,
+                 uint64_t seed, double temperature, double top_p, const uint8_t* mask,
+                 int* out_tokens, orc_stats* stats, double* draft_logits_out,
+                 double* verify_logits_out) {
+    return orc_generate_ex(m, prompt, n_prompt, n_new, K, mode, seed, temperature, top_p, mask, out_tokens,
+                           stats, draft_logits_out, verify_logits_out, NULL, NULL, NULL);
 }
