@@ -93,6 +93,7 @@ typedef struct {
     float verify_ms;   /* GPU time in verification stages incl. acceptance */
     float total_ms;    /* GPU time of the decode loop (prefill excluded) */
     long long kernel_launches; /* CUDA kernels launched by the decode loop */
+    float gamma;       /* draft-exit threshold after the last round (0 when the exit is off) */
 } ssd_stats;
 
 /* Creates a handle: validates the shape, takes the weights (see
@@ -117,6 +118,23 @@ int ssd_set_skip(ssd_handle* h, const uint8_t* mask, int n_sublayers);
  * same transform gives the draft distribution q.  temperature > 0,
  * 0 < top_p <= 1.  Errors: INVALID_ARG. */
 int ssd_set_sampling(ssd_handle* h, float temperature, float top_p);
+
+/* Adaptive draft exit (Sec. 3.4, Eqs. 2-4; Algorithms 3 / 4 of App. G).
+ * enable = 1: within a round, the draft whose confidence - the largest
+ * probability of the distribution it was chosen from (softmax of the draft
+ * logits in greedy mode, the temperature / nucleus distribution in sampling
+ * mode) - falls below gamma is the round's last draft (it is still
+ * verified).  After every verification that had drafts, with AR_e =
+ * accepted / drafted of that round:
+ *   AR <- beta1 AR + (1 - beta1) AR_e       (beta1 = 0 at the first update)
+ *   gamma <- beta2 gamma + (1 - beta2) (gamma + eps if AR <= alpha, else gamma - eps)
+ * gamma starts at gamma0 in every ssd_generate call; beta2 = 1 keeps a static
+ * threshold.  enable = 0 (the default) drafts K tokens every round (Alg. 2).
+ * The exit keeps greedy output identical to autoregressive output.  Needs
+ * gamma0 >= 0, eps >= 0 and alpha, beta1, beta2 in [0, 1].
+ * Errors: INVALID_ARG. */
+int ssd_set_draft_exit(ssd_handle* h, int enable, float gamma0, float alpha, float eps, float beta1,
+                       float beta2);
 
 /* Prefill: runs prompt[0 .. n_prompt-2] through the full model, filling KV
  * positions [0, n_prompt-1); prompt[n_prompt-1] becomes the first round's

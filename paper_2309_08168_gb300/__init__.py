@@ -26,7 +26,7 @@ SSD_GREEDY = 0
 SSD_SAMPLE = 1
 
 # every symbol include/ssd.h declares
-EXPORTS = ("ssd_create", "ssd_set_skip", "ssd_set_sampling", "ssd_prefill", "ssd_generate",
+EXPORTS = ("ssd_create", "ssd_set_skip", "ssd_set_sampling", "ssd_set_draft_exit", "ssd_prefill", "ssd_generate",
            "ssd_debug_forward", "ssd_debug_spec_accept", "ssd_debug_time_forward", "ssd_destroy",
            "ssd_last_error", "ssd_linear_noalloc", "ssd_debug_trace_forward")
 
@@ -51,13 +51,13 @@ class ssd_stats(ctypes.Structure):
     _fields_ = [("rounds", ctypes.c_int), ("drafted", ctypes.c_int), ("accepted", ctypes.c_int),
                 ("emitted", ctypes.c_int), ("accept_rate", ctypes.c_double), ("hist", ctypes.c_int * 33),
                 ("draft_ms", ctypes.c_float), ("verify_ms", ctypes.c_float), ("total_ms", ctypes.c_float),
-                ("kernel_launches", ctypes.c_longlong)]
+                ("kernel_launches", ctypes.c_longlong), ("gamma", ctypes.c_float)]
 
     def as_dict(self) -> dict:
         return {"rounds": self.rounds, "drafted": self.drafted, "accepted": self.accepted,
                 "emitted": self.emitted, "accept_rate": self.accept_rate, "hist": list(self.hist),
                 "draft_ms": self.draft_ms, "verify_ms": self.verify_ms, "total_ms": self.total_ms,
-                "kernel_launches": self.kernel_launches}
+                "kernel_launches": self.kernel_launches, "gamma": self.gamma}
 
 
 class SSDError(RuntimeError):
@@ -75,6 +75,7 @@ def _load():
     lib.ssd_create.argtypes = [ctypes.POINTER(ssd_config), ctypes.POINTER(ssd_weights), _VP, ctypes.POINTER(H)]
     lib.ssd_set_skip.argtypes = [H, _VP, ctypes.c_int]
     lib.ssd_set_sampling.argtypes = [H, ctypes.c_float, ctypes.c_float]
+    lib.ssd_set_draft_exit.argtypes = [H, ctypes.c_int] + [ctypes.c_float] * 5
     lib.ssd_prefill.argtypes = [H, _VP, ctypes.c_int]
     lib.ssd_generate.argtypes = [H, _VP, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                  ctypes.c_uint64, _VP, ctypes.POINTER(ssd_stats)]
@@ -91,8 +92,8 @@ def _load():
     lib.ssd_destroy.restype = None
     lib.ssd_last_error.argtypes = []
     lib.ssd_last_error.restype = ctypes.c_char_p
-    for n in ("ssd_create", "ssd_set_skip", "ssd_set_sampling", "ssd_prefill", "ssd_generate",
-              "ssd_debug_forward", "ssd_debug_spec_accept", "ssd_debug_time_forward"):
+    for n in ("ssd_create", "ssd_set_skip", "ssd_set_sampling", "ssd_set_draft_exit", "ssd_prefill",
+              "ssd_generate", "ssd_debug_forward", "ssd_debug_spec_accept", "ssd_debug_time_forward"):
         getattr(lib, n).restype = ctypes.c_int
     return lib
 
@@ -128,6 +129,11 @@ def ssd_set_skip(h: int, mask) -> None:
 
 def ssd_set_sampling(h: int, temperature: float, top_p: float) -> None:
     _check(lib.ssd_set_sampling(h, temperature, top_p))
+
+
+def ssd_set_draft_exit(h: int, enable: bool, gamma0: float = 0.6, alpha: float = 0.9, eps: float = 0.01,
+                       beta1: float = 0.5, beta2: float = 0.9) -> None:
+    _check(lib.ssd_set_draft_exit(h, int(bool(enable)), gamma0, alpha, eps, beta1, beta2))
 
 
 def ssd_prefill(h: int, prompt) -> None:
@@ -279,6 +285,9 @@ class Decoder:
 
     def set_sampling(self, temperature, top_p):
         ssd_set_sampling(self.h, temperature, top_p)
+
+    def set_draft_exit(self, enable, gamma0=0.6, alpha=0.9, eps=0.01, beta1=0.5, beta2=0.9):
+        ssd_set_draft_exit(self.h, enable, gamma0, alpha, eps, beta1, beta2)
 
     def prefill(self, prompt):
         ssd_prefill(self.h, prompt)

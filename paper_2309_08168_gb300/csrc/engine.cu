@@ -97,6 +97,9 @@ struct ssd_handle {
     std::vector<void*> bufs;   // work buffers
     std::vector<uint8_t> mask;
     float temperature = 1.f, top_p = 1.f;
+    // adaptive draft exit (ssd_set_draft_exit)
+    int exit_on = 0;
+    float gamma0 = 0.f, alpha = 0.f, eps = 0.f, beta1 = 0.f, beta2 = 1.f;
 
     // device buffers
     f16* kc = nullptr;   // [L][Hkv][max_seq][hd] fp16
@@ -727,6 +730,22 @@ int ssd_set_sampling(ssd_handle* h, float temperature, float top_p) {
     return SSD_OK;
 }
 
+int ssd_set_draft_exit(ssd_handle* h, int enable, float gamma0, float alpha, float eps, float beta1,
+                       float beta2) {
+    if (!h) return fail(SSD_ERR_INVALID_ARG, "NULL handle");
+    if (enable != 0 && enable != 1) return fail(SSD_ERR_INVALID_ARG, "enable must be 0 or 1");
+    auto unit = [](float x) { return x >= 0.f && x <= 1.f; };
+    if (enable && (!(gamma0 >= 0.f) || !(eps >= 0.f) || !unit(alpha) || !unit(beta1) || !unit(beta2)))
+        return fail(SSD_ERR_INVALID_ARG, "need gamma0 >= 0, eps >= 0 and alpha, beta1, beta2 in [0, 1]");
+    h->exit_on = enable;
+    h->gamma0 = gamma0;
+    h->alpha = alpha;
+    h->eps = eps;
+    h->beta1 = beta1;
+    h->beta2 = beta2;
+    return SSD_OK;
+}
+
 int ssd_prefill(ssd_handle* h, const int32_t* prompt, int n_prompt) {
     if (!h || !prompt) return fail(SSD_ERR_INVALID_ARG, "NULL handle or prompt");
     if (n_prompt < 1) return fail(SSD_ERR_INVALID_ARG, "n_prompt must be >= 1");
@@ -792,6 +811,13 @@ int ssd_generate(ssd_handle* h, const int32_t* prompt, int n_prompt, int n_new, 
     init->inv_temperature = 1.0f / h->temperature;
     init->top_p = h->top_p;
     init->seed = (unsigned long long)seed;
+    const bool exit_on = h->exit_on && K > 0;
+    init->exit_on = exit_on;
+    init->gamma = h->gamma0;
+    init->alpha = h->alpha;
+    init->eps = h->eps;
+    init->beta1 = h->beta1;
+    init->beta2 = h->beta2;
     CUDA_TRY(cudaMemcpyAsync(h->st, init, sizeof(DecodeState), cudaMemcpyHostToDevice, h->stream), "state upload");
 
     // graphs needed by this call (captured once, replayed every round)
@@ -812,15 +838,30 @@ int ssd_generate(ssd_handle* h, const int32_t* prompt, int n_prompt, int n_new, 
     int emitted = 0, round = 0;
     while (emitted < n_new) {
         const int Kd = std::min(K, n_new - emitted - 1);
+        // (graphs are captured while the stream is idle)
         cudaGraphExec_t g_verify = nullptr;
         int verify_launches = 0;
-        int rc = get_graph(h, G_VERIFY, Kd + 1, mode, &g_verify, &verify_launches);
-        if (rc) return rc;
-        launches += (long long)Kd * draft_launches + verify_launches;
+        if (!(exit_on && Kd > 0)) {
+            int rc = get_graph(h, G_VERIFY, Kd + 1, mode, &g_verify, &verify_launches);
+            if (rc) return rc;
+        }
         cudaEvent_t* ev = &h->events[2 + 3 * (size_t)round];
         CUDA_TRY(cudaEventRecord(ev[0], h->stream), "event");
         for (int j = 0; j < Kd; ++j) CUDA_TRY(cudaGraphLaunch(g_draft, h->stream), "draft step");
         CUDA_TRY(cudaEventRecord(ev[1], h->stream), "event");
+        // with the draft exit the round's draft count is known on the device
+        // only: read it before choosing the verification's row count
+        int Kv = Kd;
+        if (exit_on && Kd > 0) {
+            CUDA_TRY(cudaMemcpyAsync(h->emitted_host + 2, &h->st->j, sizeof(int), cudaMemcpyDeviceToHost, h->stream),
+                     "draft count read");
+            CUDA_TRY(cudaStreamSynchronize(h->stream), "drafting stage");
+            Kv = h->emitted_host[2];
+            if (Kv < 1 || Kv > Kd) return fail(SSD_ERR_CUDA, "decode state corrupted");
+            int rc = get_graph(h, G_VERIFY, Kv + 1, mode, &g_verify, &verify_launches);
+            if (rc) return rc;
+        }
+        launches += (long long)Kd * draft_launches + verify_launches;
         CUDA_TRY(cudaGraphLaunch(g_verify, h->stream), "verification step");
         CUDA_TRY(cudaEventRecord(ev[2], h->stream), "event");
         CUDA_TRY(cudaMemcpyAsync(h->emitted_host, &h->st->emitted, sizeof(int), cudaMemcpyDeviceToHost, h->stream),
@@ -861,6 +902,7 @@ int ssd_generate(ssd_handle* h, const int32_t* prompt, int n_prompt, int n_new, 
         stats->verify_ms = vm;
         stats->total_ms = t;
         stats->kernel_launches = launches;
+        stats->gamma = exit_on ? s->gamma : 0.f;
     }
     return SSD_OK;
 }

@@ -1104,7 +1104,7 @@ template <int R, int HD>
 __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams p) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     __shared__ float r_s[kMaxRows];
-    __shared__ int s_pos0, s_fail;
+    __shared__ int s_pos0, s_fail, s_skip;
     __shared__ unsigned s_seq;
     constexpr int S = GemmSmem<R>::S;
     __shared__ __align__(8) uint64_t full[S];   // TMA completion per stage
@@ -1119,6 +1119,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         else pos0 = p.st->len;
         s_pos0 = pos0;
         s_fail = 0;
+        // a draft step after the round's drafting stage ended (draft exit): no work
+        s_skip = p.src == SRC_DRAFT && *(volatile int*)&p.st->exited;
         s_seq = *(volatile unsigned*)p.seq;  // this forward's number (advanced by CTA 0 below)
         for (int st = 0; st < S; ++st) {
             mbar_init(full + st, 1);
@@ -1129,6 +1131,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         if (p.trace && blockIdx.x == 0) p.trace[0] = globaltimer();
     }
     __syncthreads();
+    if (s_skip) return;
     // every stage starts empty: each consumer warp releases it once
     if (threadIdx.x < kConsumers && (threadIdx.x & 31) == 0)
         for (int st = 0; st < S; ++st) mbar_arrive(empty + st);

@@ -262,17 +262,30 @@ __device__ int sample_row(const float* s, int V, float u, float* red, int* redi)
 // ---------------------------------------------------------------------------
 // kernels
 // ---------------------------------------------------------------------------
-// greedy drafting: d_{j+1} = argmax of the draft logits
+// greedy drafting: d_{j+1} = argmax of the draft logits.  With the draft
+// exit on, the draft's confidence max softmax = 1 / sum_x exp(l_x - l_max)
+// below gamma ends the round's drafting (Sec. 3.4; the draft is kept); a
+// drafting stage that has ended adds nothing.
 __global__ void __launch_bounds__(kRowThreads) greedy_draft_kernel(const float* __restrict__ logits,
                                                                    int V, DecodeState* st) {
     pdl_launch_dependents();
     pdl_wait();
     __shared__ float redf[33];
     __shared__ int redi[34];
+    if (st->exited) return;
     int best = block_argmax(logits, V, redf, redi);
+    bool stop = false;
+    if (st->exit_on) {
+        const float lmax = logits[best];
+        float s = 0.f;
+        for (int i = threadIdx.x; i < V; i += kRowThreads) s += expf(logits[i] - lmax);
+        s = block_sum(s, redf);
+        stop = 1.f / s < st->gamma;
+    }
     if (threadIdx.x == 0) {
         st->drafts[st->j] = best;
         st->j = st->j + 1;
+        if (stop) st->exited = 1;
     }
 }
 
@@ -289,6 +302,16 @@ __device__ void emit_round(DecodeState* st, int n, int y, int Kd, int* out_token
     st->accepted += n;
     st->hist[n] += 1;
     st->j = 0;
+    // adaptive draft exit: Eqs. 2-4 after a verification that had drafts
+    if (st->exit_on && Kd > 0) {
+        const float ar_e = (float)n / (float)Kd;
+        const float b1 = st->exit_updates == 0 ? 0.f : st->beta1;
+        st->ar_smooth = b1 * st->ar_smooth + (1.f - b1) * ar_e;
+        const float gt = st->ar_smooth <= st->alpha ? st->gamma + st->eps : st->gamma - st->eps;
+        st->gamma = st->beta2 * st->gamma + (1.f - st->beta2) * gt;
+        st->exit_updates += 1;
+    }
+    st->exited = 0;
 }
 
 // greedy verification: one CTA per row computes argmax p_m; the last CTA
@@ -328,15 +351,22 @@ __global__ void __launch_bounds__(kRowThreads) sample_draft_kernel(const float* 
     pdl_wait();
     __shared__ float red[33];
     __shared__ int redi[34];
+    if (st->exited) return;  // the round's drafting stage has ended
     const int j = st->j;
     nucleus_row(logits, V, st->inv_temperature, st->top_p, s, red);
     float* q = q_rows + (size_t)j * V;
-    for (int i = threadIdx.x; i < V; i += kRowThreads) q[i] = s[i];
+    float qmax = 0.f;
+    for (int i = threadIdx.x; i < V; i += kRowThreads) {
+        q[i] = s[i];
+        qmax = fmaxf(qmax, s[i]);
+    }
+    const bool stop = st->exit_on && block_max(qmax, red) < st->gamma;  // confidence = max q (Sec. 3.4)
     const float u = uniform01(st->seed, st->len + j + 1, 0);
     int d = sample_row(s, V, u, red, redi);
     if (threadIdx.x == 0) {
         st->drafts[j] = d;
         st->j = j + 1;
+        if (stop) st->exited = 1;
     }
 }
 

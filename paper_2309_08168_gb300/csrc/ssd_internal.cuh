@@ -37,6 +37,12 @@ struct DecodeState {
     float top_p;
     unsigned long long seed;
     int err;        // device-side error code (0 = none)
+    // adaptive draft exit (Sec. 3.4, Eqs. 2-4); exit_on = 0: off
+    int exit_on;
+    int exited;     // the current round's drafting stage has ended
+    int exit_updates;
+    float gamma, ar_smooth;
+    float alpha, eps, beta1, beta2;
 };
 
 // ---------------------------------------------------------------------------

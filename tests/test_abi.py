@@ -26,7 +26,7 @@ def ssd():
 
 def test_exports_every_declared_symbol(ssd):
     names = _declared()
-    assert len(names) == 12
+    assert len(names) == 13
     assert sorted(ssd.EXPORTS) == names
     lib = ctypes.CDLL(ssd.LIB_PATH)
     for n in names:
@@ -34,13 +34,14 @@ def test_exports_every_declared_symbol(ssd):
 
 
 def test_struct_layouts_match_header(ssd):
-    # ssd_config: 8 ints + 2 floats; ssd_stats: 4 ints, double, 33 ints, 3 floats
+    # ssd_config: 8 ints + 2 floats; ssd_stats: 4 ints, double, 33 ints, 3 floats, long long, float
     assert ctypes.sizeof(ssd.ssd_config) == 40
     assert ctypes.sizeof(ssd.ssd_weights) == 8 * 12 + 8
     assert ssd.ssd_stats.accept_rate.offset == 16
     assert ssd.ssd_stats.hist.offset == 24
     assert ssd.ssd_stats.total_ms.offset == 24 + 33 * 4 + 8
     assert ssd.ssd_stats.kernel_launches.offset == 168
+    assert ssd.ssd_stats.gamma.offset == 176 and ctypes.sizeof(ssd.ssd_stats) == 184
 
 
 def _cfg(ssd, **kw):
@@ -83,6 +84,7 @@ def test_null_handle_calls_fail_cleanly(ssd):
     lib = ssd.lib
     assert lib.ssd_set_skip(None, None, 0) == ssd.SSD_ERR_INVALID_ARG
     assert lib.ssd_set_sampling(None, 1.0, 1.0) == ssd.SSD_ERR_INVALID_ARG
+    assert lib.ssd_set_draft_exit(None, 1, 0.6, 0.9, 0.01, 0.5, 0.9) == ssd.SSD_ERR_INVALID_ARG
     assert lib.ssd_prefill(None, None, 1) == ssd.SSD_ERR_INVALID_ARG
     assert lib.ssd_generate(None, None, 0, 1, 0, 0, 0, None, None) == ssd.SSD_ERR_INVALID_ARG
     lib.ssd_destroy(None)
