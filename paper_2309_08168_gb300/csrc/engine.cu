@@ -180,7 +180,7 @@ const bf16* next_norm(const ssd_handle* h, int s, bool draft) {
 // TMA descriptors.  Index layout: layer l's wq wk wv wo w_gate w_up w_down at
 // 7l + 0..6, lm_head at 7L, then the input-plane maps at 7L + 1 + buf * 4 + cls
 // with buf 0 = normalised rows (K = d), 1 = attention output (K = H*hd),
-// 2 = SwiGLU output (K = ffn) and cls = rows per plane 1 | 8 | 12 | 16, then the
+// 2 = SwiGLU output (K = ffn) and cls = rows per plane 1 | 4 | 8 | 12 | 16, then the
 // K and V cache maps.
 // ---------------------------------------------------------------------------
 size_t trace_words(const ssd_handle* h) { return (size_t)kTraceCtas + 8 * (size_t)h->n_sms; }
@@ -259,7 +259,7 @@ int build_tmaps(ssd_handle* h) {
     if (!rc) rc = encode_weight(enc, &maps[7 * L], h->lm_head, d, c.vocab);
     const bf16* planes[3] = {h->xn_hi, h->at_hi, h->ac_hi};
     const int widths[3] = {d, qd, c.ffn};
-    const int rows[kPlaneClasses] = {1, 8, 12, 16};
+    const int rows[kPlaneClasses] = {1, 4, 8, 12, 16};
     for (int b = 0; b < 3 && !rc; ++b)
         for (int cls = 0; cls < kPlaneClasses && !rc; ++cls)
             rc = encode_planes(enc, &maps[tmap_x(h, b, cls)], planes[b], widths[b], rows[cls]);

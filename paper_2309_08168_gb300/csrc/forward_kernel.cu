@@ -274,7 +274,9 @@ constexpr int kAttnSegChunks = 2;
 // After the ring: the consumers' scratch - split-K reduction buffers of a
 // projection, or (same bytes: one op at a time) q / scores of attention.
 // index of the input-plane tensor map of R rows
-__host__ __device__ constexpr int plane_cls(int R) { return R == 1 ? 0 : (R == 8 ? 1 : (R == 12 ? 2 : 3)); }
+__host__ __device__ constexpr int plane_cls(int R) {
+    return R == 1 ? 0 : (R == 4 ? 1 : (R == 8 ? 2 : (R == 12 ? 3 : 4)));
+}
 
 template <int R>
 struct GemmSmem {
@@ -1231,35 +1233,44 @@ int configure_fwd() {
 }  // namespace
 
 size_t forward_smem_bytes(int M) {
-    const int R = fwd_plane_rows(M);
-    return R == 1 ? GemmSmem<1>::BYTES
-                  : (R == 8 ? GemmSmem<8>::BYTES : (R == 12 ? GemmSmem<12>::BYTES : GemmSmem<16>::BYTES));
+    switch (fwd_plane_rows(M)) {
+        case 1: return GemmSmem<1>::BYTES;
+        case 4: return GemmSmem<4>::BYTES;
+        case 8: return GemmSmem<8>::BYTES;
+        case 12: return GemmSmem<12>::BYTES;
+        default: return GemmSmem<16>::BYTES;
+    }
 }
-
 
 int forward_configure() {
     int e = 0;
     e = e ? e : configure_fwd<1, 64>();
+    e = e ? e : configure_fwd<4, 64>();
     e = e ? e : configure_fwd<8, 64>();
     e = e ? e : configure_fwd<12, 64>();
     e = e ? e : configure_fwd<16, 64>();
     e = e ? e : configure_fwd<1, 128>();
+    e = e ? e : configure_fwd<4, 128>();
     e = e ? e : configure_fwd<8, 128>();
     e = e ? e : configure_fwd<12, 128>();
     e = e ? e : configure_fwd<16, 128>();
     return e;
 }
 
+template <int HD>
+int launch_hd(const FwdParams& p, int grid, cudaStream_t s) {
+    switch (fwd_plane_rows(p.M)) {
+        case 1: return launch_fwd<1, HD>(p, grid, s);
+        case 4: return launch_fwd<4, HD>(p, grid, s);
+        case 8: return launch_fwd<8, HD>(p, grid, s);
+        case 12: return launch_fwd<12, HD>(p, grid, s);
+        default: return launch_fwd<16, HD>(p, grid, s);
+    }
+}
+
 int launch_forward(const FwdParams& p, int head_dim, int grid, cudaStream_t s) {
-    const int R = fwd_plane_rows(p.M);
-    if (head_dim == 128)
-        return R == 1 ? launch_fwd<1, 128>(p, grid, s)
-             : R == 8 ? launch_fwd<8, 128>(p, grid, s)
-             : R == 12 ? launch_fwd<12, 128>(p, grid, s) : launch_fwd<16, 128>(p, grid, s);
-    if (head_dim == 64)
-        return R == 1 ? launch_fwd<1, 64>(p, grid, s)
-             : R == 8 ? launch_fwd<8, 64>(p, grid, s)
-             : R == 12 ? launch_fwd<12, 64>(p, grid, s) : launch_fwd<16, 64>(p, grid, s);
+    if (head_dim == 128) return launch_hd<128>(p, grid, s);
+    if (head_dim == 64) return launch_hd<64>(p, grid, s);
     return (int)cudaErrorInvalidValue;
 }
 

@@ -19,6 +19,9 @@ constexpr int kAttnChunk = 64;    // KV positions per attention CTA (absolute ch
 constexpr int kAttnThreads = 256;
 constexpr int kStreamKC = 256;    // k per streaming-GEMM work unit (64 rows x 256 = 32 KB of weights)
 constexpr int kTraceUnits = 1024, kTraceCtas = 1280;  // offsets in FwdParams::trace
+// rows per input plane of a forward of M rows (the plane classes)
+constexpr int fwd_plane_rows(int M) { return M == 1 ? 1 : (M <= 4 ? 4 : (M <= 8 ? 8 : (M <= 12 ? 12 : 16))); }
+constexpr int kPlaneClasses = 5;
 
 // ---------------------------------------------------------------------------
 // device state of the decode loop (one per handle, in device memory)
@@ -97,7 +100,7 @@ struct GemmArgs {
     // 64-wide k-box.
     int wide;
     const void* tm_w[3];  // w0, w1, w2
-    const void* tm_x[4];  // input planes for R = 1 | 8 | 12 | 16
+    const void* tm_x[kPlaneClasses];  // input planes for R = 1 | 4 | 8 | 12 | 16
 };
 
 // ---------------------------------------------------------------------------
@@ -173,11 +176,6 @@ int gemm_configure();
 int launch_gemm(int epi, const GemmArgs& a, cudaStream_t s);
 size_t gemm_smem_bytes(int kc, int M);
 constexpr int gemm_half_rows(int M) { return M <= 8 ? 8 : 16; }  // padded rows of x_hi (and of x_lo)
-// R of the forward kernel: input-plane rows per op (1 | 8 | 12 | 16)
-constexpr int fwd_plane_rows(int M) { return M == 1 ? 1 : (M <= 8 ? 8 : (M <= 12 ? 12 : 16)); }
-constexpr int kPlaneClasses = 4;
-
-
 
 // src for launch_embed
 enum EmbedSrc { SRC_TOKENS = 0, SRC_DRAFT = 1, SRC_VERIFY = 2 };
