@@ -15,6 +15,9 @@
   * With an empty skip set every draft is accepted, so each round's AR_e is
     1 > alpha and gamma falls by (1 - beta2) * eps per round: the final gamma
     has a closed form in the number of rounds.
+  * In sampling mode the exit depends only on the draft distribution, so the
+    first emitted token still follows the target's nucleus distribution p_0
+    (chi-square over seeds, with a threshold that makes the exit point vary).
 """
 import numpy as np
 import pytest
@@ -130,3 +133,31 @@ def test_empty_mask_gamma_closed_form(micro):
         if k > 0:
             g -= 0.1 * 0.01
         assert got == pytest.approx(g, abs=1e-12)
+
+
+def test_sampling_with_exit_keeps_the_first_token_law():
+    """The exit decision depends only on the draft distribution q, so the
+    speculative-sampling guarantee is untouched: the first emitted token
+    still follows the target's nucleus distribution p_0 (Alg. 4)."""
+    from scipy.stats import chi2
+    w = micro_workload(vocab=16, n_prompt=3)
+    wts = synth.host_weights(w, seed=21)
+    pr = synth.prompt(3, seed=2, vocab=w.vocab)
+    o = oracle.Oracle(w, wts, max_seq=12)
+    o.prefill(pr)
+    p0 = oracle.nucleus_probs(o.forward(int(pr[-1]), 2) * 40.0, 1.0, 0.95)
+    T = 2500
+    toks = np.empty(T, dtype=np.int64)
+    keff = np.empty(T, dtype=np.int64)
+    for s in range(T):
+        out, st = o.generate(pr, 5, 3, mode=1, seed=5000 + s, temperature=1 / 40, top_p=0.95, mask=w.mask(),
+                             draft_exit=(0.8, 0.9, 0.0, 0.5, 1.0))
+        toks[s] = out[0]
+        keff[s] = st["keff"][0]
+    assert len(set(keff.tolist())) > 1  # the first round's exit point varies with the draws
+    counts = np.bincount(toks, minlength=w.vocab)
+    keep = p0 * T >= 5
+    assert counts[~keep].sum() <= max(10, 3 * p0[~keep].sum() * T)
+    exp = p0[keep] * T
+    stat = ((counts[keep] - exp) ** 2 / exp).sum() + 0.0
+    assert chi2.sf(stat, max(1, keep.sum() - 1)) > 1e-4, (counts, p0 * T)
