@@ -114,3 +114,18 @@ def test_exit_static_threshold_draft_counts_vs_oracle(tiny_setup, mode):
     if np.array_equal(toks, ref):
         assert abs(st["drafted"] - rst["drafted"]) <= max(4, rst["drafted"] // 8)
     dec.close()
+
+
+def test_exit_bad_arguments(tiny_setup):
+    import paper_2309_08168_gb300 as ssd
+    w, hw, dw = tiny_setup
+    dec = decoder(w, dw, 160)
+    for bad in ((-0.1, 0.9, 0.01, 0.5, 0.9), (0.6, 1.5, 0.01, 0.5, 0.9), (0.6, 0.9, -0.01, 0.5, 0.9),
+                (0.6, 0.9, 0.01, 1.5, 0.9), (0.6, 0.9, 0.01, 0.5, -0.1)):
+        with pytest.raises(ssd.SSDError):
+            dec.set_draft_exit(True, *bad)
+    dec.set_draft_exit(False, -1.0, 2.0, -1.0, 3.0, 3.0)  # parameters are not checked when off
+    prompt = synth.prompt(w.n_prompt, seed=0, vocab=w.vocab)
+    a, st = dec.generate(prompt, 8, 4)
+    assert st["gamma"] == 0.0
+    dec.close()
