@@ -99,6 +99,8 @@ def lib():
         L.orc_exit_update.argtypes = [ctypes.POINTER(OrcExitState), ctypes.POINTER(OrcExit), ctypes.c_double]
         L.orc_softmax_max.argtypes = [_P, ctypes.c_int]
         L.orc_softmax_max.restype = ctypes.c_double
+        L.orc_set_threads.argtypes = [ctypes.c_int]
+        L.orc_get_threads.restype = ctypes.c_int
         L.orc_rmsnorm.argtypes = [_P, _P, ctypes.c_int, ctypes.c_double, _P]
         L.orc_rope.argtypes = [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_double]
         L.orc_philox4x32_10.argtypes = [_P, _P, _P]
@@ -302,6 +304,15 @@ def exit_update(state, params, ar_e):
     st = OrcExitState(*state)
     lib().orc_exit_update(ctypes.byref(st), ctypes.byref(OrcExit(1, *map(float, params))), float(ar_e))
     return st.gamma, st.ar, st.e
+
+
+def set_threads(n: int) -> None:
+    """OpenMP threads of the oracle (timing only; results do not depend on it)."""
+    lib().orc_set_threads(int(n))
+
+
+def get_threads() -> int:
+    return int(lib().orc_get_threads())
 
 
 def softmax_max(logits):

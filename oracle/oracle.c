@@ -59,6 +59,7 @@
  *     gamma0 for every generation.
  */
 #include <math.h>
+#include <omp.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -102,6 +103,11 @@ typedef struct {
 /* ------------------------------------------------------------------------ */
 /* small helpers                                                             */
 /* ------------------------------------------------------------------------ */
+
+/* OpenMP threads of the row-parallel loops (timing runs; results do not
+ * depend on it: every dot product is summed in k order by one thread). */
+void orc_set_threads(int n) { omp_set_num_threads(n > 0 ? n : 1); }
+int orc_get_threads(void) { return omp_get_max_threads(); }
 
 double orc_bf16_to_f64(uint16_t b) {
     uint32_t u = ((uint32_t)b) << 16;
