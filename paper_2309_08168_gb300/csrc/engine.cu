@@ -127,8 +127,7 @@ struct ssd_handle {
     float* p_rows = nullptr;
     float* q_rows = nullptr;
     float* partial = nullptr;
-    unsigned* counters = nullptr;  // [gemm tiles | attention kv heads | accept]
-    int gemm_counters = 0;
+    unsigned* counters = nullptr;  // [attention kv heads | accept] arrival counters
     float* attn_part = nullptr;
     int n_chunks = 0;
     float2* rope = nullptr;
@@ -293,7 +292,6 @@ GemmArgs proj_args(ssd_handle* h, int N, int K, int n_tiles, const bf16* x_hi, c
     a.x_hi = x_hi;
     a.x_lo = x_lo;
     a.partial = h->partial;
-    a.counters = h->counters;
     a.st = h->st;
     a.err = &h->st->err;
     a.inv_dim = 1.0f / (float)h->cfg.d_model;
@@ -340,7 +338,7 @@ std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
             t.q = h->q;
             t.tm_k = h->tmaps + tmap_kv(h, 0); t.tm_v = h->tmaps + tmap_kv(h, 1); t.kv_z0 = l * c.n_kv_heads;
             t.out_hi = h->at_hi; t.out_lo = h->at_lo;
-            t.part = h->attn_part; t.counters = h->counters + h->gemm_counters;
+            t.part = h->attn_part; t.counters = h->counters;
             t.n_heads = c.n_heads; t.n_kv_heads = c.n_kv_heads; t.head_dim = c.head_dim;
             t.max_seq = c.max_seq; t.n_chunks = h->n_chunks;
             t.scale = 1.0f / std::sqrt((float)c.head_dim); t.st = h->st; t.err = &h->st->err;
@@ -445,7 +443,7 @@ double forward_weight_bytes(const ssd_handle* h, bool draft, bool gemm_only) {
     return b;
 }
 
-unsigned* accept_counter(ssd_handle* h) { return h->counters + h->gemm_counters + h->cfg.n_kv_heads; }
+unsigned* accept_counter(ssd_handle* h) { return h->counters + h->cfg.n_kv_heads; }
 
 int step_launches(ssd_handle* h, int kind, int M, int mode, int* n_launch) {
     const int V = h->cfg.vocab;
@@ -633,14 +631,11 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
     h->p_down = make_plan(c.ffn, (d + kTileRows - 1) / kTileRows);
     h->p_head = make_plan(d, (c.vocab + kTileRows - 1) / kTileRows);
     size_t part = 0;
-    int tiles = 0;
     for (const GemmPlan* p : {&h->p_qkv, &h->p_o, &h->p_gu, &h->p_down, &h->p_head}) {
         const int K = p == &h->p_o ? qd : (p == &h->p_down ? c.ffn : d);
         const size_t chunks = (size_t)(K + kStreamKC - 1) / kStreamKC;
         part = std::max(part, chunks * kMaxRows * p->n_tiles * kTileRows);
-        tiles = std::max(tiles, p->n_tiles);
     }
-    h->gemm_counters = tiles;
     h->n_chunks = (c.max_seq + kAttnChunk - 1) / kAttnChunk;
     const int G = c.n_heads / c.n_kv_heads;
 
@@ -659,7 +654,7 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
         (rc = dalloc(h, &h->p_rows, (size_t)kMaxRows * V, &B)) ||
         (rc = dalloc(h, &h->q_rows, (size_t)kMaxRows * V, &B)) ||
         (rc = dalloc(h, &h->partial, 2 * part, &B)) ||  // tagged 64-bit words in the forward kernel
-        (rc = dalloc(h, &h->counters, (size_t)tiles + c.n_kv_heads + 4, &B)) ||
+        (rc = dalloc(h, &h->counters, (size_t)c.n_kv_heads + 4, &B)) ||
         (rc = dalloc(h, &h->attn_part, (size_t)c.n_kv_heads * h->n_chunks * G * kMaxRows * (HD + 2), &B)) ||
         (rc = dalloc(h, &h->rope, (size_t)c.max_seq * (HD / 2), &B)) ||
         (rc = dalloc(h, &h->tok, (size_t)c.max_seq + kMaxRows, &B)) ||
@@ -694,7 +689,7 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
         cudaError_t e = cudaMemcpy(h->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice);
         if (e != cudaSuccess) return bail(fail(SSD_ERR_CUDA, std::string("rope table: ") + cudaGetErrorString(e)));
     }
-    cudaError_t e = cudaMemsetAsync(h->counters, 0, ((size_t)tiles + c.n_kv_heads + 4) * sizeof(unsigned), h->stream);
+    cudaError_t e = cudaMemsetAsync(h->counters, 0, ((size_t)c.n_kv_heads + 4) * sizeof(unsigned), h->stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(h->st, 0, sizeof(DecodeState), h->stream);
     // barrier counter and forward sequence number; split-K slots hold no
     // valid tag (a tag is never 0: GEMM ops have an op index >= 1)
@@ -757,8 +752,8 @@ int ssd_prefill(ssd_handle* h, const int32_t* prompt, int n_prompt) {
     CUDA_TRY(cudaMemsetAsync(&h->st->err, 0, sizeof(int), h->stream), "error flag reset");
     // arrival counters are left at zero by every completed op; after a timed-out
     // forward they may not be, so a new prompt starts from clean counters
-    CUDA_TRY(cudaMemsetAsync(h->counters, 0, ((size_t)h->gemm_counters + h->cfg.n_kv_heads) * sizeof(unsigned),
-                             h->stream), "counter reset");
+    CUDA_TRY(cudaMemsetAsync(h->counters, 0, (size_t)h->cfg.n_kv_heads * sizeof(unsigned), h->stream),
+             "counter reset");
     if (n_prompt > 1)
         CUDA_TRY(cudaMemcpyAsync(h->tok, prompt, sizeof(int) * (n_prompt - 1), cudaMemcpyHostToDevice, h->stream),
                  "prompt upload");

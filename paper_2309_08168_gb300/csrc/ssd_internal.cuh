@@ -66,7 +66,7 @@ struct GemmArgs {
     int M;               // activation rows (1..16)
     float* partial;      // split-K partials: gemm.cu [ksplit][M][n_tiles*64] floats; forward
                          // kernel [n_tiles][n_chunks][16][64] tagged 64-bit words
-    unsigned* counters;  // [n_tiles] arrival counters of gemm.cu (left at zero)
+    unsigned* counters;  // gemm.cu: [n_tiles] arrival counters (left at zero); unused by the forward kernel
     // epilogue operands
     float* out_f32;      // EPI_LOGITS: [M][ldo]; EPI_RESID: residual h [M][ldo]
     int ldo;
