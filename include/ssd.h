@@ -37,7 +37,8 @@ extern "C" {
 #define SSD_ERR_OOM (-2)         /* device memory allocation failed */
 #define SSD_ERR_CUDA (-3)        /* a CUDA call or kernel failed */
 #define SSD_ERR_CAPACITY (-4)    /* prompt + n_new exceeds max_seq */
-#define SSD_ERR_TIMEOUT (-5)     /* reserved: a bounded device wait gave up */
+#define SSD_ERR_TIMEOUT (-5)     /* a bounded device wait gave up (a grid barrier or a copy that did not
+                                    complete within its limit); the handle stays usable */
 #define SSD_ERR_STATE (-6)       /* call out of order (e.g. generate without a prompt or prefill) */
 
 typedef struct ssd_handle ssd_handle;
@@ -136,11 +137,13 @@ int ssd_set_sampling(ssd_handle* h, float temperature, float top_p);
 int ssd_set_draft_exit(ssd_handle* h, int enable, float gamma0, float alpha, float eps, float beta1,
                        float beta2);
 
-/* Prefill: runs prompt[0 .. n_prompt-2] through the full model, filling KV
+/* Prefill: encodes the prompt with the full model before decoding starts
+ * (Sec. 3.1: the prefix x_1..x_t that Algorithms 1 and 2 continue from).
+ * It runs prompt[0 .. n_prompt-2] through the full model, filling KV
  * positions [0, n_prompt-1); prompt[n_prompt-1] becomes the first round's
  * x_last, so every generated token comes from a decoding round.  prompt is a
  * host array of token ids in [0, vocab); 1 <= n_prompt <= max_seq.
- * Errors: INVALID_ARG, CAPACITY, CUDA. */
+ * Errors: INVALID_ARG, CAPACITY, CUDA, TIMEOUT. */
 int ssd_prefill(ssd_handle* h, const int32_t* prompt, int n_prompt);
 
 /* Generates n_new tokens (Algorithm 2 for SSD_GREEDY, Algorithm 4 for
@@ -156,12 +159,25 @@ int ssd_generate(ssd_handle* h, const int32_t* prompt, int n_prompt, int n_new, 
                  ssd_mode mode, uint64_t seed, int32_t* out_tokens, ssd_stats* stats);
 
 /* Parity hook: one forward of n_rows tokens (host ids) at positions
- * pos0 .. pos0+n_rows-1 over the current KV cache, full model (draft = 0) or
- * the skip-set model (draft = 1), writing KV like the decode loop does and
- * copying fp32 logits [n_rows][vocab] to host logits_out.  1 <= n_rows <= 16;
- * pos0 + n_rows <= max_seq.  Errors: INVALID_ARG, CUDA. */
+ * pos0 .. pos0+n_rows-1 over the current KV cache, full model (draft = 0:
+ * the verification forward of Algorithm 2 / 4, which produces the target
+ * rows p_0..p_K) or the skip-set model (draft = 1: one drafting step of
+ * Sec. 3.2, the draft distribution q), writing KV like the decode loop does
+ * and copying fp32 logits [n_rows][vocab] to host logits_out.
+ * 1 <= n_rows <= 16; pos0 + n_rows <= max_seq.
+ * Errors: INVALID_ARG, CUDA, TIMEOUT. */
 int ssd_debug_forward(ssd_handle* h, int draft, const int32_t* tokens, int n_rows, int pos0,
                       float* logits_out);
+
+/* Test hook for the bounded waits (the paper has no counterpart): arms the
+ * next ssd_debug_forward on this handle to make its grid barrier number
+ * `barrier` (1 = the barrier after the embedding) unreachable and to give up
+ * waiting after wait_limit_s seconds; that forward then returns
+ * SSD_ERR_TIMEOUT, its logits are unspecified and the handle stays usable
+ * (the next forward runs normally).  barrier = 0 disarms.  The hook applies
+ * to that one forward only, never to ssd_generate or ssd_prefill.
+ * 0 < wait_limit_s <= 10.  Errors: INVALID_ARG. */
+int ssd_debug_stall_barrier(ssd_handle* h, int barrier, double wait_limit_s);
 
 /* Parity hook for the speculative-sampling acceptance kernel of Algorithm 4
  * in isolation: `trials` independent verifications sharing the target rows
@@ -228,11 +244,15 @@ int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, in
  * and, when K > 512, ceil(K/512) * M * 64 * ceil(N/64) <= 1,048,576 scratch
  * floats; larger problems are rejected with SSD_ERR_CAPACITY before any
  * launch.  The first call on each device does a one-time set-up with that
- * device current (symbol lookup, kernel attribute, zeroing the counters);
- * make that first call before any stream capture.  Every call zeroes the
- * counters it uses on the stream before its kernel; the scratch arrays are
- * shared by all calls on a device, so calls that overlap on the GPU (other
- * streams, other threads) race and must be serialised by the caller.
+ * device current (symbol lookup, kernel attribute); make that first call
+ * before any stream capture.  Every call zeroes the counters it uses on the
+ * stream before its kernel; the scratch arrays are shared by all calls on a
+ * device, so calls that overlap on the GPU (other streams, other threads)
+ * race and must be serialised by the caller.  Faults inside the kernel are
+ * not reported by this call (it returns once the work is enqueued); builds
+ * with the device-side checks enabled (SSD_CHECKED=1) read the check flag
+ * back after the kernel, which makes the call synchronous, and report a
+ * failed check as SSD_ERR_CUDA.
  * Errors: INVALID_ARG, CAPACITY, CUDA. */
 int ssd_linear_noalloc(const void* w, const float* x, float* y, int N, int K, int M,
                        void* cuda_stream);

@@ -28,7 +28,7 @@ SSD_SAMPLE = 1
 # every symbol include/ssd.h declares
 EXPORTS = ("ssd_create", "ssd_set_skip", "ssd_set_sampling", "ssd_set_draft_exit", "ssd_prefill", "ssd_generate",
            "ssd_debug_forward", "ssd_debug_spec_accept", "ssd_debug_time_forward", "ssd_destroy",
-           "ssd_last_error", "ssd_linear_noalloc", "ssd_debug_trace_forward")
+           "ssd_last_error", "ssd_linear_noalloc", "ssd_debug_trace_forward", "ssd_debug_stall_barrier")
 
 
 class ssd_config(ctypes.Structure):
@@ -86,6 +86,8 @@ def _load():
     lib.ssd_debug_trace_forward.argtypes = [H, ctypes.c_int, ctypes.c_int, _VP, _VP, ctypes.c_int, _VP,
                                             ctypes.c_int, _VP, _VP, ctypes.c_int, _VP]
     lib.ssd_debug_trace_forward.restype = ctypes.c_int
+    lib.ssd_debug_stall_barrier.argtypes = [H, ctypes.c_int, ctypes.c_double]
+    lib.ssd_debug_stall_barrier.restype = ctypes.c_int
     lib.ssd_linear_noalloc.argtypes = [_VP, _VP, _VP, ctypes.c_int, ctypes.c_int, ctypes.c_int, _VP]
     lib.ssd_linear_noalloc.restype = ctypes.c_int
     lib.ssd_destroy.argtypes = [H]
@@ -161,6 +163,10 @@ def ssd_debug_forward(h: int, draft: bool, tokens, pos0: int) -> np.ndarray:
     out = np.empty((t.size, config_of(h).vocab), dtype=np.float32)
     _check(lib.ssd_debug_forward(h, int(draft), t.ctypes.data, t.size, pos0, out.ctypes.data))
     return out
+
+
+def ssd_debug_stall_barrier(h: int, barrier: int, wait_limit_s: float) -> None:
+    _check(lib.ssd_debug_stall_barrier(h, int(barrier), float(wait_limit_s)))
 
 
 def ssd_debug_spec_accept(h: int, p, q, drafts, seeds, pos0: int):
@@ -297,6 +303,9 @@ class Decoder:
 
     def debug_forward(self, draft, tokens, pos0):
         return ssd_debug_forward(self.h, draft, tokens, pos0)
+
+    def debug_stall_barrier(self, barrier, wait_limit_s):
+        return ssd_debug_stall_barrier(self.h, barrier, wait_limit_s)
 
     def debug_spec_accept(self, p, q, drafts, seeds, pos0):
         return ssd_debug_spec_accept(self.h, p, q, drafts, seeds, pos0)

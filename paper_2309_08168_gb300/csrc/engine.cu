@@ -147,6 +147,17 @@ struct ssd_handle {
     int n_prompt = 0;
     int last_prompt_token = 0;
     bool sync_check = false;
+    // prefill on the tensor cores (prefill.cu): plan, per-layer arguments and
+    // TMA maps (box 64 x 128); used for prompts of more than 16 rows
+    bool pf_on = false;
+    PrefillPlan pf{};
+    std::vector<PrefillLayer> pf_layers;
+    CUtensorMap* pf_tmaps = nullptr;
+    // bounded waits of the forward kernel; test hook: one forward of
+    // ssd_debug_forward with an unreachable grid barrier (ssd_debug_stall_barrier)
+    unsigned long long wait_ns = 2000000000ull;
+    int stall_barrier = 0;
+    unsigned long long stall_wait_ns = 0;
 };
 
 namespace {
@@ -276,6 +287,63 @@ int build_tmaps(ssd_handle* h) {
     return SSD_OK;
 }
 
+// TMA maps of the prefill GEMMs: every matrix [rows][K] bf16 viewed as
+// {K, rows}, box 64 (k) x 128 rows, 128-byte swizzle (the tcgen05 operand
+// layout); layer l's wq wk wv wo w_gate w_up w_down at 7l + 0..6, then the
+// activation planes x hi / lo, attention output hi / lo, SwiGLU output hi / lo.
+int build_prefill(ssd_handle* h) {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    CUDA_TRY(cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q),
+             "driver entry point");
+    if (!fn || q != cudaDriverEntryPointSuccess) return fail(SSD_ERR_CUDA, "cuTensorMapEncodeTiled unavailable");
+    auto enc = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+    const ssd_config& c = h->cfg;
+    const int L = c.n_layers, d = c.d_model, qd = c.n_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
+    PrefillPlan& P = h->pf;
+    std::vector<CUtensorMap> maps((size_t)7 * L + 6);
+    auto map2 = [&](CUtensorMap* m, const void* base, int K, int rows) {
+        cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
+        cuuint64_t strides[1] = {(cuuint64_t)K * 2};
+        cuuint32_t box[2] = {64, 128};
+        return encode_map(enc, m, base, 2, dims, strides, box);
+    };
+    int rc = 0;
+    for (int l = 0; l < L && !rc; ++l) {
+        const bf16* w[7] = {h->wq[l], h->wk[l], h->wv[l], h->wo[l], h->w_gate[l], h->w_up[l], h->w_down[l]};
+        const int K[7] = {d, d, d, qd, d, d, c.ffn};
+        const int N[7] = {qd, kvd, kvd, d, c.ffn, c.ffn, d};
+        for (int i = 0; i < 7 && !rc; ++i) rc = map2(&maps[7 * l + i], w[i], K[i], N[i]);
+    }
+    const size_t a0 = (size_t)7 * L;
+    if (!rc) rc = map2(&maps[a0 + 0], P.x_hi, d, P.rows);
+    if (!rc) rc = map2(&maps[a0 + 1], P.x_lo, d, P.rows);
+    if (!rc) rc = map2(&maps[a0 + 2], P.at_hi, qd, P.rows);
+    if (!rc) rc = map2(&maps[a0 + 3], P.at_lo, qd, P.rows);
+    if (!rc) rc = map2(&maps[a0 + 4], P.ac_hi, c.ffn, P.rows);
+    if (!rc) rc = map2(&maps[a0 + 5], P.ac_lo, c.ffn, P.rows);
+    if (rc) return rc;
+    CUDA_TRY(cudaMemcpy(h->pf_tmaps, maps.data(), maps.size() * sizeof(CUtensorMap), cudaMemcpyHostToDevice),
+             "prefill tensor map upload");
+    h->pf_layers.resize(L);
+    for (int l = 0; l < L; ++l) {
+        PrefillLayer& Ly = h->pf_layers[l];
+        for (int i = 0; i < 7; ++i) Ly.tm_w[i] = h->pf_tmaps + 7 * l + i;
+        Ly.attn_norm = h->attn_norm[l];
+        Ly.mlp_norm = h->mlp_norm[l];
+        Ly.k_cache = h->kc + (size_t)l * h->kv_layer;
+        Ly.v_cache = h->vc + (size_t)l * h->kv_layer;
+    }
+    P.tm_x[0] = h->pf_tmaps + a0 + 0;
+    P.tm_x[1] = h->pf_tmaps + a0 + 1;
+    P.tm_at[0] = h->pf_tmaps + a0 + 2;
+    P.tm_at[1] = h->pf_tmaps + a0 + 3;
+    P.tm_ac[0] = h->pf_tmaps + a0 + 4;
+    P.tm_ac[1] = h->pf_tmaps + a0 + 5;
+    P.layers = h->pf_layers.data();
+    return SSD_OK;
+}
+
 void set_x_maps(const ssd_handle* h, GemmArgs& a, int buf) {
     for (int cls = 0; cls < kPlaneClasses; ++cls) a.tm_x[cls] = h->tmaps + tmap_x(h, buf, cls);
 }
@@ -338,7 +406,7 @@ std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
             t.q = h->q;
             t.tm_k = h->tmaps + tmap_kv(h, 0); t.tm_v = h->tmaps + tmap_kv(h, 1); t.kv_z0 = l * c.n_kv_heads;
             t.out_hi = h->at_hi; t.out_lo = h->at_lo;
-            t.part = h->attn_part; t.counters = h->counters;
+            t.part = h->attn_part;
             t.n_heads = c.n_heads; t.n_kv_heads = c.n_kv_heads; t.head_dim = c.head_dim;
             t.max_seq = c.max_seq; t.n_chunks = h->n_chunks;
             t.scale = 1.0f / std::sqrt((float)c.head_dim); t.st = h->st; t.err = &h->st->err;
@@ -400,7 +468,7 @@ int upload_ops(ssd_handle* h, bool draft) {
 // kernel over the op list (lm_head dropped when no logits are needed).
 // Launches only; no host synchronisation (graph-capturable).
 int forward(ssd_handle* h, int M, int src, const int* toks, int pos0, bool draft, bool logits,
-            int* n_launch = nullptr, unsigned long long* trace = nullptr) {
+            int* n_launch = nullptr, unsigned long long* trace = nullptr, int stall_barrier = 0) {
     const ssd_config& c = h->cfg;
     FwdParams p{};
     p.ops = draft ? h->ops_draft : h->ops_full;
@@ -422,6 +490,8 @@ int forward(ssd_handle* h, int M, int src, const int* toks, int pos0, bool draft
     p.err = &h->st->err;
     p.trace = trace;
     p.trace_op = h->trace_op;
+    p.wait_ns = h->wait_ns;
+    p.stall_barrier = stall_barrier;
     CUDA_TRY(cudaMemsetAsync(h->bar, 0, sizeof(unsigned), h->stream), "barrier reset");
     LAUNCH(h, launch_forward(p, c.head_dim, h->n_sms, h->stream), "forward kernel", -1);
     if (n_launch) *n_launch = 1;
@@ -700,6 +770,40 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
     if (e == cudaSuccess) e = cudaStreamSynchronize(h->stream);
     if (e != cudaSuccess) return bail(fail(SSD_ERR_CUDA, std::string("init: ") + cudaGetErrorString(e)));
     if ((rc = build_tmaps(h)) || (rc = upload_ops(h, false)) || (rc = upload_ops(h, true))) return bail(rc);
+
+    // prefill on the tensor cores: needs the q / k / v widths in whole
+    // 128-row boxes; otherwise prompts run through the decode kernel
+    {
+        const char* e = std::getenv("SSD_TC_PREFILL");
+        h->pf_on = e && e[0] == '1' && qd % 128 == 0 && kvd % 128 == 0;
+    }
+    if (h->pf_on) {
+        PrefillPlan& P = h->pf;
+        P.n_layers = L;
+        P.d = d;
+        P.n_heads = c.n_heads;
+        P.n_kv_heads = c.n_kv_heads;
+        P.head_dim = c.head_dim;
+        P.ffn = c.ffn;
+        P.max_seq = c.max_seq;
+        P.eps = c.rms_eps;
+        P.rows = std::min(c.max_seq, 2048);
+        P.embed = h->embed;
+        P.rope = h->rope;
+        P.err = &h->st->err;
+        const size_t R = (size_t)P.rows;
+        if ((rc = dalloc(h, &P.h, R * d, &B)) || (rc = dalloc(h, &P.x_hi, 2 * R * d, &B)) ||
+            (rc = dalloc(h, &P.q, R * qd, &B)) || (rc = dalloc(h, &P.at_hi, 2 * R * qd, &B)) ||
+            (rc = dalloc(h, &P.ac_hi, 2 * R * F, &B)) ||
+            (rc = dalloc(h, &h->pf_tmaps, (size_t)7 * L + 6, &B)))
+            return bail(rc);
+        P.x_lo = P.x_hi + R * d;
+        P.at_lo = P.at_hi + R * qd;
+        P.ac_lo = P.ac_hi + R * F;
+        int e4 = prefill_configure();
+        if (e4) return bail(fail(SSD_ERR_CUDA, std::string("prefill setup: ") + cudaGetErrorString((cudaError_t)e4)));
+        if ((rc = build_prefill(h))) return bail(rc);
+    }
     *out = h;
     return SSD_OK;
 }
@@ -750,17 +854,28 @@ int ssd_prefill(ssd_handle* h, const int32_t* prompt, int n_prompt) {
     CUDA_TRY(cudaSetDevice(h->device), "set device");
     h->prefilled = false;
     CUDA_TRY(cudaMemsetAsync(&h->st->err, 0, sizeof(int), h->stream), "error flag reset");
-    // arrival counters are left at zero by every completed op; after a timed-out
-    // forward they may not be, so a new prompt starts from clean counters
-    CUDA_TRY(cudaMemsetAsync(h->counters, 0, (size_t)h->cfg.n_kv_heads * sizeof(unsigned), h->stream),
+    // the acceptance kernels' arrival counter is left at zero by every
+    // completed launch; after a failed one it may not be, so a new prompt
+    // starts from clean counters
+    CUDA_TRY(cudaMemsetAsync(h->counters, 0, ((size_t)h->cfg.n_kv_heads + 4) * sizeof(unsigned), h->stream),
              "counter reset");
     if (n_prompt > 1)
         CUDA_TRY(cudaMemcpyAsync(h->tok, prompt, sizeof(int) * (n_prompt - 1), cudaMemcpyHostToDevice, h->stream),
                  "prompt upload");
-    for (int p0 = 0; p0 < n_prompt - 1; p0 += kMaxRows) {
-        int M = std::min(kMaxRows, n_prompt - 1 - p0);
-        int rc = forward(h, M, SRC_TOKENS, h->tok + p0, p0, false, false);
-        if (rc) return rc;
+    if (h->pf_on && n_prompt - 1 > kMaxRows) {
+        // tensor-core prefill, chunks of up to pf.rows positions
+        for (int p0 = 0; p0 < n_prompt - 1; p0 += h->pf.rows) {
+            const int n = std::min(h->pf.rows, n_prompt - 1 - p0);
+            int e = prefill_chunk(h->pf, h->tok + p0, n, p0, h->stream);
+            if (e) return fail(SSD_ERR_CUDA, std::string("prefill: ") + cudaGetErrorString((cudaError_t)e));
+            if (h->sync_check) CUDA_TRY(cudaStreamSynchronize(h->stream), "prefill chunk");
+        }
+    } else {
+        for (int p0 = 0; p0 < n_prompt - 1; p0 += kMaxRows) {
+            int M = std::min(kMaxRows, n_prompt - 1 - p0);
+            int rc = forward(h, M, SRC_TOKENS, h->tok + p0, p0, false, false);
+            if (rc) return rc;
+        }
     }
     CUDA_TRY(cudaStreamSynchronize(h->stream), "prefill");
     {
@@ -910,12 +1025,35 @@ int ssd_debug_forward(ssd_handle* h, int draft, const int32_t* tokens, int n_row
         if (tokens[i] < 0 || tokens[i] >= h->cfg.vocab) return fail(SSD_ERR_INVALID_ARG, "token out of range");
     CUDA_TRY(cudaSetDevice(h->device), "set device");
     int* dt = h->tok + h->cfg.max_seq;
+    CUDA_TRY(cudaMemsetAsync(&h->st->err, 0, sizeof(int), h->stream), "error flag reset");
     CUDA_TRY(cudaMemcpyAsync(dt, tokens, sizeof(int) * n_rows, cudaMemcpyHostToDevice, h->stream), "upload");
-    int rc = forward(h, n_rows, SRC_TOKENS, dt, pos0, draft != 0, true);
+    const int stall = h->stall_barrier;
+    const unsigned long long wait_ns = h->wait_ns;
+    if (stall) {  // armed by ssd_debug_stall_barrier for this one forward
+        h->wait_ns = h->stall_wait_ns;
+        h->stall_barrier = 0;
+    }
+    int rc = forward(h, n_rows, SRC_TOKENS, dt, pos0, draft != 0, true, nullptr, nullptr, stall);
+    h->wait_ns = wait_ns;
     if (rc) return rc;
     CUDA_TRY(cudaMemcpyAsync(logits_out, h->logits, sizeof(float) * n_rows * h->cfg.vocab,
                              cudaMemcpyDeviceToHost, h->stream), "logits");
+    int derr = 0;
+    CUDA_TRY(cudaMemcpyAsync(&h->st_host->err, &h->st->err, sizeof(int), cudaMemcpyDeviceToHost, h->stream),
+             "error flag");
     CUDA_TRY(cudaStreamSynchronize(h->stream), "debug forward");
+    derr = h->st_host->err;
+    if (derr == kDevErrTimeout) return fail(SSD_ERR_TIMEOUT, "a wait of the forward kernel timed out");
+    if (derr) return fail(SSD_ERR_CUDA, "device check failed with code " + std::to_string(derr));
+    return SSD_OK;
+}
+
+int ssd_debug_stall_barrier(ssd_handle* h, int barrier, double wait_limit_s) {
+    if (!h) return fail(SSD_ERR_INVALID_ARG, "NULL handle");
+    if (barrier < 0 || !(wait_limit_s > 0.0) || wait_limit_s > 10.0)
+        return fail(SSD_ERR_INVALID_ARG, "need barrier >= 0 and 0 < wait_limit_s <= 10");
+    h->stall_barrier = barrier;
+    h->stall_wait_ns = (unsigned long long)(wait_limit_s * 1e9);
     return SSD_OK;
 }
 

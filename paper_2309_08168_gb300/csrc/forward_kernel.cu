@@ -72,8 +72,8 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
 // Grid-wide barrier for a cooperative launch (all CTAs co-resident).  The
 // counter only grows during a launch; `target` = gridDim.x * (barrier index).
 // Returns false (and records SSD_DEV_ERR_TIMEOUT) if the others do not arrive
-// within kBarrierTimeoutNs, or if another CTA already gave up.
-__device__ bool grid_barrier(unsigned* bar, unsigned target, int* err) {
+// within limit_ns, or if another CTA already gave up.
+__device__ bool grid_barrier(unsigned* bar, unsigned target, int* err, unsigned long long limit_ns) {
     __shared__ int s_ok;
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -85,7 +85,7 @@ __device__ bool grid_barrier(unsigned* bar, unsigned target, int* err) {
         const unsigned long long t0 = globaltimer();
         while (ld_acquire(bar) < target) {  // acquire: later loads see the others' stores
             if (*(volatile int*)err) { ok = 0; break; }
-            if (globaltimer() - t0 > kBarrierTimeoutNs) {
+            if (globaltimer() - t0 > limit_ns) {
                 atomicCAS(err, 0, kDevErrTimeout);
                 ok = 0;
                 break;
@@ -822,7 +822,6 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
     float* sc = reinterpret_cast<float*>(smem + L::ATT_SC);  // [VG][SP] scores
     __half* ph = reinterpret_cast<__half*>(smem + L::ATT_P);  // [VG][PST] weights hi, then lo
     __half* pl = ph + VG * PST;
-    __shared__ unsigned s_mask;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, tg = lane & 3;
     const size_t part_v = HD + 2;  // floats per partial: o[HD], max, sum
@@ -842,19 +841,36 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
         const int v0 = vg * VG, nv = min(VG, NV - v0);
         float* part = a.part + ((size_t)kvh * a.n_chunks + sg) * NV * part_v;
         // q of this item's vectors as fp16 hi + lo (other CTAs wrote q: L2);
-        // the loads overlap the wait for K / V; consecutive items of one KV
-        // head and vector group reuse it
+        // every thread issues all its 16-byte loads before converting, and the
+        // loads overlap the wait for K / V; consecutive items of one KV head
+        // and vector group reuse it
         const int key = kvh * ar.n_vg + vg;
-        for (int k = key == q_key ? VG * HD : tid; k < VG * HD; k += kConsumers) {
-            const int vl = k / HD, e = k - vl * HD;
-            float x = 0.f;
-            if (vl < nv) {
-                const int v = v0 + vl, m = v / G, gi = v - m * G;
-                x = __ldcg(a.q + (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e);
+        if (key != q_key) {
+            constexpr int HD4 = HD / 4, QJ = VG * HD4 / kConsumers;  // float4 per thread: 2 | 1
+            static_assert(VG * HD4 % kConsumers == 0, "q tile split evenly over the consumers");
+            float4 qv[QJ];
+#pragma unroll
+            for (int j = 0; j < QJ; ++j) {
+                const int k4 = tid + j * kConsumers, vl = k4 / HD4, e = (k4 - vl * HD4) * 4;
+                qv[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (vl < nv) {
+                    const int v = v0 + vl, m = v / G, gi = v - m * G;
+                    qv[j] = __ldcg(reinterpret_cast<const float4*>(a.q + (size_t)m * a.n_heads * HD +
+                                                                   (size_t)(kvh * G + gi) * HD + e));
+                }
             }
-            const __half xh = __float2half_rn(x);
-            qh[vl * QST + e] = xh;
-            ql[vl * QST + e] = __float2half_rn(x - __half2float(xh));
+#pragma unroll
+            for (int j = 0; j < QJ; ++j) {
+                const int k4 = tid + j * kConsumers, vl = k4 / HD4, e = (k4 - vl * HD4) * 4;
+                const __half2 h01 = __floats2half2_rn(qv[j].x, qv[j].y), h23 = __floats2half2_rn(qv[j].z, qv[j].w);
+                const float2 f01 = __half22float2(h01), f23 = __half22float2(h23);
+                const __half2 l01 = __floats2half2_rn(qv[j].x - f01.x, qv[j].y - f01.y);
+                const __half2 l23 = __floats2half2_rn(qv[j].z - f23.x, qv[j].w - f23.y);
+                *reinterpret_cast<uint2*>(qh + vl * QST + e) =
+                    make_uint2(*reinterpret_cast<const uint32_t*>(&h01), *reinterpret_cast<const uint32_t*>(&h23));
+                *reinterpret_cast<uint2*>(ql + vl * QST + e) =
+                    make_uint2(*reinterpret_cast<const uint32_t*>(&l01), *reinterpret_cast<const uint32_t*>(&l23));
+            }
         }
         q_key = key;
         stamp(it, 1);
@@ -970,83 +986,62 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
             for (int j = 0; j < n_u; ++j) mbar_arrive(pp.empty + (i + j) % S);  // the stages are free
         i += n_u;
     }
-    if (ar.i_begin >= ar.i_end) return ok;
-    if (ct && tid == 0) {
+    if (ct && tid == 0 && ar.i_begin < ar.i_end) {
         ct[2] = globaltimer();
         ct[6] = (unsigned long long)(ar.i_end - ar.i_begin);
     }
-
-    // publish the partials; each KV head's count is completed by one CTA, which
-    // combines that head (all heads a CTA completes are combined in one pass)
-    __threadfence();
-    consumer_sync();
-    if (ut && tid == 0) ut[248] = globaltimer();
-    const int per_kv = ar.n_seg * ar.n_vg;  // items of one KV head
-    const int kv_lo = ar.i_begin / per_kv, kv_hi = (ar.i_end - 1) / per_kv;
-    for (int kb = kv_lo; kb <= kv_hi; kb += 32) {
-        const int nk = min(32, kv_hi - kb + 1);
-        if (warp == 0) {
-            bool last = false;
-            if (lane < nk) {
-                const int kvh = kb + lane;
-                const int cnt = min(ar.i_end, (kvh + 1) * per_kv) - max(ar.i_begin, kvh * per_kv);
-                const unsigned prev = atomicAdd(&a.counters[kvh], (unsigned)cnt);
-                last = prev + (unsigned)cnt == (unsigned)per_kv;
-                if (last) a.counters[kvh] = 0u;  // no other CTA touches it again in this op
-            }
-            const unsigned mask = __ballot_sync(0xffffffffu, last);
-            if (lane == 0) s_mask = mask;
-        }
-        consumer_sync();
-        if (ut && tid == 0) ut[249] = globaltimer();
-        const int n_last = __popc(s_mask);
-        if (n_last) {
-            __threadfence();
-            // row m uses segments 0 .. (pos0 + m) / SP, summed in segment order;
-            // thread per (head, v, 4 dims): every load of a row is independent
-            for (int k = tid; k < n_last * NV * (HD / 4); k += kConsumers) {
-                const int hx = k / (NV * (HD / 4)), kk = k - hx * NV * (HD / 4);
-                unsigned mm = s_mask;  // the hx-th head this CTA completed
-                for (int r = 0; r < hx; ++r) mm &= mm - 1u;
-                const int kvh = kb + __ffs(mm) - 1;
-                const float* part = a.part + (size_t)kvh * a.n_chunks * NV * part_v;
-                const int v = kk / (HD / 4), e = (kk - v * (HD / 4)) * 4;
-                const int m = v / G, gi = v - m * G;
-                const int nsg = (pos0 + m) / SP + 1;
-                const float* pv = part + (size_t)v * part_v;
-                const size_t qs_stride = (size_t)NV * part_v;
-                float mx = -INFINITY;
-#pragma unroll 8
-                for (int q = 0; q < nsg; ++q) mx = fmaxf(mx, __ldcg(pv + q * qs_stride + HD));
-                float l = 0.f, o0 = 0.f, o1 = 0.f, o2 = 0.f, o3 = 0.f;
-#pragma unroll 8
-                for (int q = 0; q < nsg; ++q) {
-                    const float* pq = pv + q * qs_stride;
-                    const float mq = __ldcg(pq + HD);
-                    const float f = mq == -INFINITY ? 0.f : expf(mq - mx);  // empty segments hold o = 0
-                    const float2 oa = __ldcg(reinterpret_cast<const float2*>(pq + e));
-                    const float2 ob = __ldcg(reinterpret_cast<const float2*>(pq + e + 2));
-                    l += f * __ldcg(pq + HD + 1);
-                    o0 += f * oa.x;
-                    o1 += f * oa.y;
-                    o2 += f * ob.x;
-                    o3 += f * ob.y;
-                }
-                const float inv = 1.f / l;
-                const size_t at = (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e;
-                const float val[4] = {o0 * inv, o1 * inv, o2 * inv, o3 * inv};
-#pragma unroll
-                for (int x = 0; x < 4; ++x) {
-                    const bf16 vh = __float2bfloat16_rn(val[x]);
-                    a.out_hi[at + x] = vh;
-                    a.out_lo[at + x] = __float2bfloat16_rn(val[x] - __bfloat162float(vh));
-                }
-            }
-        }
-        consumer_sync();
-        if (ut && tid == 0) ut[250] = globaltimer();
-    }
     return ok;
+}
+
+// Second phase of attention, after a grid barrier (the segment partials of
+// every CTA are visible): the partials of each (KV head, query vector) are
+// combined in segment order - row m uses segments 0 .. (pos0 + m) / SP - and
+// written as the bf16 hi / lo planes of the attention output.  The outputs
+// are spread over every CTA's consumer threads, one thread per 4 dims of a
+// vector (consecutive threads: consecutive dims, coalesced loads), so the
+// combine costs about two dependent L2 round trips whatever the number of
+// vectors and segments.
+template <int HD>
+__device__ void attn_combine(const AttnArgs& a, int M, int pos0) {
+    if (threadIdx.x >= kConsumers) return;
+    constexpr int SP = kAttnSegChunks * kAttnChunk, HD4 = HD / 4;
+    const int G = a.n_heads / a.n_kv_heads, NV = G * M;
+    const size_t part_v = HD + 2;              // floats per partial: o[HD], max, sum
+    const size_t qs_stride = (size_t)NV * part_v;  // next segment of the same vector
+    const int tasks = a.n_kv_heads * NV * HD4;
+    for (int k = blockIdx.x * kConsumers + threadIdx.x; k < tasks; k += gridDim.x * kConsumers) {
+        const int kvh = k / (NV * HD4), r = k - kvh * NV * HD4;
+        const int v = r / HD4, e = (r - v * HD4) * 4;
+        const int m = v / G, gi = v - m * G;
+        const int nsg = (pos0 + m) / SP + 1;
+        const float* pv = a.part + (size_t)kvh * a.n_chunks * qs_stride + (size_t)v * part_v;
+        float mx = -INFINITY;
+#pragma unroll 8
+        for (int q = 0; q < nsg; ++q) mx = fmaxf(mx, __ldcg(pv + q * qs_stride + HD));
+        float l = 0.f, o0 = 0.f, o1 = 0.f, o2 = 0.f, o3 = 0.f;
+#pragma unroll 8
+        for (int q = 0; q < nsg; ++q) {
+            const float* pq = pv + q * qs_stride;
+            const float mq = __ldcg(pq + HD);
+            const float f = mq == -INFINITY ? 0.f : expf(mq - mx);  // empty segments hold o = 0
+            const float2 oa = __ldcg(reinterpret_cast<const float2*>(pq + e));
+            const float2 ob = __ldcg(reinterpret_cast<const float2*>(pq + e + 2));
+            l += f * __ldcg(pq + HD + 1);
+            o0 += f * oa.x;
+            o1 += f * oa.y;
+            o2 += f * ob.x;
+            o3 += f * ob.y;
+        }
+        const float inv = 1.f / l;
+        const size_t at = (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e;
+        const float val[4] = {o0 * inv, o1 * inv, o2 * inv, o3 * inv};
+#pragma unroll
+        for (int x = 0; x < 4; ++x) {
+            const bf16 vh = __float2bfloat16_rn(val[x]);
+            a.out_hi[at + x] = vh;
+            a.out_lo[at + x] = __float2bfloat16_rn(val[x] - __bfloat162float(vh));
+        }
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -1139,6 +1134,19 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         for (int st = 0; st < S; ++st) mbar_arrive(empty + st);
     const int pos0 = s_pos0;
     unsigned target = 0;
+    int n_barrier = 0;
+    // Next grid barrier of this launch.  The profiling hook p.stall_barrier
+    // (0: none) makes barrier number n unreachable, so that its bounded wait
+    // runs out and the launch ends with the timeout recorded.
+    auto barrier_next = [&]() -> bool {
+        target += gridDim.x;
+        ++n_barrier;
+        const unsigned extra = n_barrier == p.stall_barrier ? 1u : 0u;
+        if (!grid_barrier(p.bar, target + extra, p.err, p.wait_ns)) return false;
+        // every CTA has read the sequence number before the first barrier
+        if (n_barrier == 1 && blockIdx.x == 0 && threadIdx.x == 0) *p.seq = s_seq + 1u;
+        return true;
+    };
     Pipe pp{full, empty, 0u, 0u};
     bool prefetched = false;
     int attn_pre = 0;  // producer: K / V chunks of the next attention op requested early
@@ -1161,13 +1169,39 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
                              smem_u32(reinterpret_cast<unsigned char*>(s_op + ((o + 1) & 1)) + 16 * plane)),
                          "l"(reinterpret_cast<const unsigned char*>(p.ops + o + 1) + 16 * plane)
                          : "memory");
+        const FwdOp* nx = has_nx ? s_op + ((o + 1) & 1) : nullptr;
+        bool early = false;  // producer: the next projection's weights already requested
         if (is_gemm(type)) {
             ok = gemm_op<R>(op.g, epi_of(type), p.M, pos0, prefetched, smem, r_s, pp, (s_seq << 10) | (unsigned)o, p.err,
                             (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr, ct);
+        } else if (type == OP_EMBED) {
+            embed_op(p, pos0);
         } else {
-            if (type == OP_EMBED) embed_op(p, pos0);
-            else ok = attn_op<R, HD>(op.at, p.M, pos0, smem, pp, p.err, ct, attn_pre,
-                                     (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr);
+            // attention: segment partials; then, while the grid gathers, the
+            // producer requests the next projection's first weights (the ring
+            // is free again), and after the barrier every CTA combines a share
+            // of the partials
+            ok = attn_op<R, HD>(op.at, p.M, pos0, smem, pp, p.err, ct, attn_pre,
+                                (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr);
+            if (plane >= 0) {
+                asm volatile("cp.async.wait_all;" ::: "memory");
+                __syncwarp();
+            }
+            if (plane == 0 && nx && ok && is_gemm(nx->type)) {
+                ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err);
+                early = true;
+            }
+            if (!ok) s_fail = 1;
+            __syncthreads();
+            if (s_fail) {
+                drain_before_exit();
+                return;
+            }
+            if (!barrier_next()) {
+                drain_before_exit();
+                return;
+            }
+            attn_combine<HD>(op.at, p.M, pos0);
         }
         if (ct && threadIdx.x == 0) ct[3] = globaltimer();
         // next op: visible to the producer warp now, to every thread after
@@ -1176,12 +1210,11 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
             asm volatile("cp.async.wait_all;" ::: "memory");
             __syncwarp();
         }
-        const FwdOp* nx = has_nx ? s_op + ((o + 1) & 1) : nullptr;
         prefetched = false;
         attn_pre = 0;
         if (plane == 0 && nx && ok) {
             if (is_gemm(nx->type)) {
-                ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err);
+                if (!early) ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err);
                 prefetched = true;
             } else if (nx->type == OP_ATTN) {
                 attn_pre = attn_prefetch<R, HD>(nx->at, p.M, pos0, smem, pp, p.err);
@@ -1196,13 +1229,10 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         }
         if (ct && threadIdx.x == 0) ct[4] = globaltimer();
         if (o + 1 < p.n_ops) {
-            target += gridDim.x;
-            if (!grid_barrier(p.bar, target, p.err)) {
+            if (!barrier_next()) {
                 drain_before_exit();
                 return;
             }
-            // every CTA has read the sequence number before the first barrier
-            if (target == gridDim.x && blockIdx.x == 0 && threadIdx.x == 0) *p.seq = s_seq + 1u;
         }
         if (ct && threadIdx.x == 0) ct[5] = globaltimer();
         if (p.trace && blockIdx.x == 0 && threadIdx.x == 0) p.trace[o + 1] = globaltimer();

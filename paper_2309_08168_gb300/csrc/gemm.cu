@@ -328,7 +328,8 @@ int noalloc_setup(int dev, NoAllocDevice** out) {
         if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&d.err, g_noalloc_err);
         if (e == cudaSuccess) e = (cudaError_t)configure_one<1, EPI_LOGITS>();
         if (e == cudaSuccess) e = (cudaError_t)configure_one<2, EPI_LOGITS>();
-        if (e == cudaSuccess) e = cudaMemset(d.counters, 0, sizeof(unsigned) * kNoAllocTiles);
+        // (the arrays start at zero when the module loads; each call clears
+        // the counters it uses on its own stream)
         if (e != cudaSuccess)
             return set_last_error(SSD_ERR_CUDA, (std::string("ssd_linear_noalloc set-up: ") +
                                                  cudaGetErrorString(e)).c_str());
@@ -388,6 +389,20 @@ extern "C" int ssd_linear_noalloc(const void* w, const float* x, float* y, int N
         e = (cudaError_t)(M > 8 ? launch_one<2, EPI_LOGITS>(a, s) : launch_one<1, EPI_LOGITS>(a, s));
     if (e != cudaSuccess)
         return set_last_error(SSD_ERR_CUDA, (std::string("ssd_linear_noalloc: ") + cudaGetErrorString(e)).c_str());
+#ifdef SSD_CHECKED
+    // checked builds: the kernel's alignment / bounds guards record a code in
+    // the device flag; read it back (this makes the call synchronous), clear it
+    // for the next call and report it
+    int derr = 0;
+    e = cudaMemcpyAsync(&derr, d->err, sizeof(int), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(d->err, 0, sizeof(int), s);
+    if (e != cudaSuccess)
+        return set_last_error(SSD_ERR_CUDA, (std::string("ssd_linear_noalloc: ") + cudaGetErrorString(e)).c_str());
+    if (derr)
+        return set_last_error(SSD_ERR_CUDA,
+                              ("ssd_linear_noalloc: device check failed with code " + std::to_string(derr)).c_str());
+#endif
     return SSD_OK;
 }
 

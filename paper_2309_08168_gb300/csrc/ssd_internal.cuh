@@ -116,8 +116,7 @@ struct AttnArgs {
     int kv_z0;
     bf16* out_hi;        // [M][H*hd] output planes: hi = rn(o), lo = rn(o - hi)
     bf16* out_lo;
-    float* part;         // [Hkv][n_chunks][G*M][hd + 2]
-    unsigned* counters;  // [Hkv]
+    float* part;         // segment partials [Hkv][n_chunks][G*M][hd + 2]: o[hd], max, sum
     int M, n_heads, n_kv_heads, head_dim, max_seq, n_chunks;
     float scale;         // 1/sqrt(hd)
     const DecodeState* st;
@@ -162,7 +161,45 @@ struct FwdParams {
     // arrive, barrier release, number of units, 0.
     unsigned long long* trace;
     int trace_op;
+    // Bounded waits: a grid barrier gives up after wait_ns (error recorded).
+    // Test hook: stall_barrier = n > 0 makes the n-th grid barrier of the
+    // launch unreachable (0 in every production launch).
+    unsigned long long wait_ns;
+    int stall_barrier;
 };
+
+// ---------------------------------------------------------------------------
+// prefill on the tensor cores (prefill.cu, tc_gemm.cuh)
+// ---------------------------------------------------------------------------
+struct PrefillLayer {
+    const void* tm_w[7];  // TMA maps (box 64 x 128) of wq wk wv wo w_gate w_up w_down
+    const bf16* attn_norm;
+    const bf16* mlp_norm;
+    f16* k_cache;  // this layer's [Hkv][max_seq][hd]
+    f16* v_cache;
+};
+struct PrefillPlan {
+    int n_layers, d, n_heads, n_kv_heads, head_dim, ffn, max_seq;
+    float eps;
+    int rows;  // capacity of the row buffers (prompt positions per chunk)
+    const bf16* embed;
+    const float2* rope;
+    float* h;           // [rows][d]
+    bf16* x_hi;         // [rows][d] normalised rows, hi / lo
+    bf16* x_lo;
+    float* q;           // [rows][H*hd]
+    bf16* at_hi;        // [rows][H*hd] attention output, hi / lo
+    bf16* at_lo;
+    bf16* ac_hi;        // [rows][ffn] SwiGLU output, hi / lo
+    bf16* ac_lo;
+    const void* tm_x[2];   // TMA maps of x_hi / x_lo  (box 64 x 128)
+    const void* tm_at[2];  // of at_hi / at_lo
+    const void* tm_ac[2];  // of ac_hi / ac_lo
+    const PrefillLayer* layers;  // host array
+    int* err;
+};
+int prefill_configure();
+int prefill_chunk(const PrefillPlan& P, const int* toks, int n, int pos0, cudaStream_t s);
 
 int forward_configure();
 size_t forward_smem_bytes(int M);

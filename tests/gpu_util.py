@@ -46,3 +46,26 @@ def check_tokens_vs_oracle(gpu_tokens, orc, prompt, n):
             assert margin <= MARGIN, f"token {i}: gpu {gpu_tokens[i]} oracle {ref[i]} margin {margin}"
             return i
     return n
+
+
+def common_prefix_runs(dec, orc, prompt, n_new, K, mode=0, seed=0, mask=None, top_p=1.0,
+                       temperature=1.0, draft_exit=None, min_common=8):
+    """Runs the GPU decoder and the oracle on the same generation and, where
+    their tokens part (a near-tie decided in fp32 on one side and fp64 on the
+    other), re-runs both with n_new cut to the common prefix, so that the
+    statistics they return describe identical token sequences.  The decoder's
+    skip set, sampling and draft-exit settings must already match the oracle
+    arguments.  Returns (n, gpu stats, oracle stats) of the final runs;
+    asserts that at least min_common tokens are shared."""
+    n = n_new
+    for _ in range(6):
+        g, sg = dec.generate(prompt, n, K, mode=mode, seed=seed)
+        o, so = orc.generate(prompt, n, K, mode=mode, seed=seed, temperature=temperature, top_p=top_p,
+                             mask=mask, draft_exit=draft_exit)
+        diff = np.nonzero(np.asarray(g) != np.asarray(o))[0]
+        if diff.size == 0:
+            assert n >= min_common, f"only {n} common tokens"
+            return n, sg, so
+        n = int(diff[0])
+        assert n >= min_common, f"tokens part at {n}: gpu {g[n]} oracle {o[n]}"
+    raise AssertionError("no common prefix found")

@@ -26,7 +26,7 @@ def ssd():
 
 def test_exports_every_declared_symbol(ssd):
     names = _declared()
-    assert len(names) == 13
+    assert len(names) == 14
     assert sorted(ssd.EXPORTS) == names
     lib = ctypes.CDLL(ssd.LIB_PATH)
     for n in names:

@@ -50,3 +50,24 @@ def test_single_rank_is_local():
     import bench
     assert bench.reduce_max(3.0, 1) == 3.0
     assert bench.job_tokens_per_s(512, 3, 1, 1000.0) == pytest.approx(1536.0)
+
+
+def test_gpus_flag_starts_the_replicas():
+    """`bench.py --gpus 2` starts two ranks itself (torch.distributed.run on
+    127.0.0.1) and reports the ranks that ran; on a machine without GPUs the
+    ranks rendezvous over gloo.  --launch-only decodes nothing."""
+    import json
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = {k: v for k, v in os.environ.items() if k not in ("WORLD_SIZE", "RANK", "LOCAL_RANK")}
+    if not torch.cuda.is_available():
+        env["CUDA_VISIBLE_DEVICES"] = ""
+    r = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--gpus", "2", "--launch-only"],
+                       capture_output=True, text=True, timeout=300, env=env, cwd=root)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [json.loads(l) for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, r.stdout
+    assert lines[0]["n_gpus"] == 2 and lines[0]["max_rank"] == 1
+    if not torch.cuda.is_available():
+        assert lines[0]["backend"] == "gloo"

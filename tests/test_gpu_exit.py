@@ -19,7 +19,7 @@ import pytest
 
 import oracle
 import synth
-from gpu_util import decoder
+from gpu_util import common_prefix_runs, decoder
 
 pytestmark = pytest.mark.gpu
 
@@ -98,21 +98,23 @@ def test_exit_empty_mask_gamma_closed_form(tiny_setup):
 
 @pytest.mark.parametrize("mode", [0, 1])
 def test_exit_static_threshold_draft_counts_vs_oracle(tiny_setup, mode):
+    """Draft counts of the GPU and of the oracle over the same tokens (the
+    common prefix of their generations), with a static threshold near the
+    drafts' typical confidence: the exit decisions are fp32 on the GPU and
+    fp64 in the oracle, so the totals agree up to decisions at the threshold."""
     w, hw, dw = tiny_setup
     g0 = _typical_confidence(w, hw)
     params = (g0, 0.9, 0.0, 0.5, 1.0)
     dec = decoder(w, dw, 160)
     dec.set_sampling(1.0, 0.95)
     dec.set_draft_exit(True, *params)
-    prompt = synth.prompt(w.n_prompt, seed=0, vocab=w.vocab)
-    toks, st = dec.generate(prompt, w.n_new, 8, mode=mode, seed=7)
+    prompt = synth.prompt(w.n_prompt, seed=2, vocab=w.vocab)
     orc = oracle.Oracle(w, hw, max_seq=160)
-    ref, rst = orc.generate(prompt, w.n_new, 8, mode=mode, seed=7, top_p=0.95, mask=w.mask(),
-                            draft_exit=params)
-    assert st["emitted"] == w.n_new == st["rounds"] + st["accepted"]
+    n, st, rst = common_prefix_runs(dec, orc, prompt, w.n_new, 8, mode=mode, seed=7, mask=w.mask(),
+                                    top_p=0.95, draft_exit=params, min_common=16)
+    assert st["emitted"] == n == st["rounds"] + st["accepted"]
     assert st["rounds"] - 1 <= st["drafted"] <= 8 * st["rounds"]
-    if np.array_equal(toks, ref):
-        assert abs(st["drafted"] - rst["drafted"]) <= max(4, rst["drafted"] // 8)
+    assert abs(st["drafted"] - rst["drafted"]) <= max(4, rst["drafted"] // 8)
     dec.close()
 
 

@@ -17,7 +17,7 @@ import pytest
 
 import oracle
 import synth
-from gpu_util import assert_logits_close, check_tokens_vs_oracle, decoder
+from gpu_util import assert_logits_close, check_tokens_vs_oracle, common_prefix_runs, decoder
 
 pytestmark = pytest.mark.gpu
 
@@ -132,18 +132,20 @@ def test_tiny_ar_matches_oracle(ssd, tiny_setup):
 
 
 def test_tiny_ssd_stats_and_oracle_rounds(ssd, tiny_setup):
-    """With identical tokens, the acceptance pattern n per round is decided by
-    draft argmaxes; compare the GPU's acceptance with the oracle's run."""
+    """The acceptance counts of the GPU and of the oracle over the same tokens
+    (the common prefix of their generations): both follow Algorithm 2, so the
+    counts agree up to draft argmaxes decided differently at near-ties (fp32
+    vs fp64)."""
     w, hw, dw = tiny_setup
     dec = decoder(w, dw, 160)
     orc = oracle.Oracle(w, hw, max_seq=160)
-    prompt = synth.prompt(w.n_prompt, seed=0, vocab=w.vocab)
-    toks, st = dec.generate(prompt, w.n_new, w.K)
-    ref, rst = orc.generate(prompt, w.n_new, w.K, mask=w.mask())
+    # prompt 2: the oracle's top-1 / top-2 margin stays above 0.0029 over all 64 tokens
+    prompt = synth.prompt(w.n_prompt, seed=2, vocab=w.vocab)
+    n, st, rst = common_prefix_runs(dec, orc, prompt, w.n_new, w.K, mask=w.mask(), min_common=16)
     assert st["drafted"] > 0 and st["accept_rate"] > 0.3
-    if np.array_equal(toks, ref):
-        # tiny margins can flip a draft argmax; totals stay close
-        assert abs(st["accepted"] - rst["accepted"]) <= max(3, rst["accepted"] // 10)
+    assert st["emitted"] == rst["emitted"] == n
+    assert abs(st["accepted"] - rst["accepted"]) <= max(3, rst["accepted"] // 10)
+    assert abs(st["rounds"] - rst["rounds"]) <= max(3, rst["rounds"] // 10)
     dec.close()
 
 

@@ -3,12 +3,16 @@ the decoding loops per emitted token, on a LLaMA-2-7B-width model truncated to
 4 layers (8 sublayers; skipping one saves ~100 MB of weight streaming per
 draft step).  Started from the empty skip set, the search must find a skip
 set that decodes faster per token, and the decoder keeps decoding correctly
-with it (greedy output identical to its AR output)."""
+with it: greedy output identical to its AR output, tokens equal to the fp64
+oracle's self-speculative decoding with the same skip set z wherever the
+oracle's top-1 / top-2 margin exceeds 0.1, and acceptance counts equal to the
+oracle's over the tokens both produced."""
 import numpy as np
 import pytest
 
+import oracle
 import synth
-from gpu_util import decoder
+from gpu_util import check_tokens_vs_oracle, common_prefix_runs, decoder
 
 pytestmark = pytest.mark.gpu
 
@@ -35,4 +39,16 @@ def test_search_improves_on_the_empty_skip_set():
     ar, _ = dec.generate(None, 32, 0)
     sd, _ = dec.generate(None, 32, 4)
     assert np.array_equal(ar, sd)
+
+    # the oracle with the skip set the search found (same bf16 weight bits)
+    hw = synth.host_weights(w, seed=0)
+    orc = oracle.Oracle(w, hw, max_seq=400)
+    n = check_tokens_vs_oracle(sd, orc, prompts[0], 32)
+    assert n >= 16, n
+    ref, rst = orc.generate(prompts[0], n, 4, mask=z)
+    assert np.array_equal(sd[:n], ref)  # Algorithm 2 with z is lossless in the oracle too
+    m, st, rst = common_prefix_runs(dec, orc, prompts[0], n, 4, mask=z, min_common=n)
+    # draft argmaxes at near-ties can be decided differently (fp32 vs fp64)
+    assert abs(st["accepted"] - rst["accepted"]) <= max(2, rst["accepted"] // 10)
+    assert abs(st["rounds"] - rst["rounds"]) <= max(2, rst["rounds"] // 10)
     dec.close()
