@@ -773,10 +773,7 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
 
     // prefill on the tensor cores: needs the q / k / v widths in whole
     // 128-row boxes; otherwise prompts run through the decode kernel
-    {
-        const char* e = std::getenv("SSD_TC_PREFILL");
-        h->pf_on = e && e[0] == '1' && qd % 128 == 0 && kvd % 128 == 0;
-    }
+    h->pf_on = qd % 128 == 0 && kvd % 128 == 0;
     if (h->pf_on) {
         PrefillPlan& P = h->pf;
         P.n_layers = L;
