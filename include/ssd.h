@@ -45,7 +45,9 @@ typedef struct ssd_handle ssd_handle;
 
 /* Model shape (LLaMA-2 decoder, Sec. 4.1 / App. B).
  *   head_dim must be 64 or 128; n_heads a multiple of n_kv_heads (GQA);
- *   d_model a multiple of 64; ffn a multiple of 16 and >= 64; 2 <= vocab <= 32768;
+ *   d_model, n_heads * head_dim and n_kv_heads * head_dim multiples of 128
+ *   (the forward kernel's 128-row tiles); ffn a multiple of 16 and >= 64;
+ *   2 <= vocab <= 32768;
  *   max_seq = KV capacity in positions (>= n_prompt + n_new).
  * Numerics: bf16 weights; fp32 residual stream, norms, softmax and
  * accumulation; activations enter each projection as bf16 hi + lo pairs;

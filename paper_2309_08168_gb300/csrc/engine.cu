@@ -67,18 +67,6 @@ int fail(int code, const std::string& msg) {
         }                                                                                       \
     } while (0)
 
-struct GemmPlan {
-    int kc = 0, ksplit = 0, n_tiles = 0;
-};
-
-GemmPlan make_plan(int K, int n_tiles) {
-    GemmPlan p;
-    p.kc = K >= 512 ? 512 : ((K + 63) / 64) * 64;
-    p.ksplit = (K + p.kc - 1) / p.kc;
-    p.n_tiles = n_tiles;
-    return p;
-}
-
 enum GraphKind { G_DRAFT = 0, G_VERIFY = 1 };
 
 }  // namespace
@@ -138,7 +126,6 @@ struct ssd_handle {
     DecodeState* st_host = nullptr;  // pinned staging
     int* emitted_host = nullptr;     // pinned
 
-    GemmPlan p_qkv, p_o, p_gu, p_down, p_head;
     std::map<int, cudaGraphExec_t> graphs;
     std::map<int, int> graph_launches;  // kernels per replay
     std::vector<cudaEvent_t> events;
@@ -217,32 +204,22 @@ int encode_map(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void
     return SSD_OK;
 }
 
-// weight matrix [rows][K] bf16.  K % 64 == 0: viewed as {64, K/64, rows} with
-// box {64, 4, 32} (a 64-row x 256-k unit is two copies); otherwise 2D with box
-// 64 (k) x 32 rows (eight copies per unit).
-int encode_weight(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* base, int K, int rows) {
-    if (K % 64 == 0) {
-        cuuint64_t dims[3] = {64, (cuuint64_t)K / 64, (cuuint64_t)rows};
-        cuuint64_t strides[2] = {128, (cuuint64_t)K * 2};
-        cuuint32_t box[3] = {64, 4, 32};
-        return encode_map(enc, m, base, 3, dims, strides, box);
-    }
+// weight matrix [rows][K] bf16 viewed as {K, rows}, box 64 (k) x box_rows:
+// one copy per 64-wide k box of a forward-kernel work unit (128 rows; 64 for
+// the gate and up halves of a SwiGLU tile), written in the 128-byte-swizzled
+// K-major layout tcgen05.mma reads
+int encode_weight(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* base, int K, int rows,
+                  int box_rows) {
     cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)rows};
     cuuint64_t strides[1] = {(cuuint64_t)K * 2};
-    cuuint32_t box[2] = {64, 32};
+    cuuint32_t box[2] = {64, (cuuint32_t)box_rows};
     return encode_map(enc, m, base, 2, dims, strides, box);
 }
 
-// input planes [2][16][K] bf16 (hi plane, lo plane).  K % 64 == 0: viewed as
-// {64, K/64, 16, 2} with box {64, 4, R, 2} (one copy per unit); otherwise 3D
-// {K, 16, 2} with box {64, R, 2} (one copy per 64-wide k-box).
+// input planes [2][16][K] bf16 (hi plane, lo plane) viewed as {K, 16, 2}, box
+// {64, R, 2}: one copy per 64-wide k box holds the R hi rows, then the R lo
+// rows, 128 bytes each (the N side of tcgen05.mma)
 int encode_planes(PFN_cuTensorMapEncodeTiled_v12000 enc, CUtensorMap* m, const void* base, int K, int R) {
-    if (K % 64 == 0) {
-        cuuint64_t dims[4] = {64, (cuuint64_t)K / 64, (cuuint64_t)kMaxRows, 2};
-        cuuint64_t strides[3] = {128, (cuuint64_t)K * 2, (cuuint64_t)K * 2 * kMaxRows};
-        cuuint32_t box[4] = {64, 4, (cuuint32_t)R, 2};
-        return encode_map(enc, m, base, 4, dims, strides, box);
-    }
     cuuint64_t dims[3] = {(cuuint64_t)K, (cuuint64_t)kMaxRows, 2};
     cuuint64_t strides[2] = {(cuuint64_t)K * 2, (cuuint64_t)K * 2 * kMaxRows};
     cuuint32_t box[3] = {64, (cuuint32_t)R, 2};
@@ -264,9 +241,10 @@ int build_tmaps(ssd_handle* h) {
         const bf16* w[7] = {h->wq[l], h->wk[l], h->wv[l], h->wo[l], h->w_gate[l], h->w_up[l], h->w_down[l]};
         const int K[7] = {d, d, d, qd, d, d, c.ffn};
         const int N[7] = {qd, kvd, kvd, d, c.ffn, c.ffn, d};
-        for (int i = 0; i < 7 && !rc; ++i) rc = encode_weight(enc, &maps[tmap_weight(l, i)], w[i], K[i], N[i]);
+        for (int i = 0; i < 7 && !rc; ++i)
+            rc = encode_weight(enc, &maps[tmap_weight(l, i)], w[i], K[i], N[i], (i == 4 || i == 5) ? 64 : kFTile);
     }
-    if (!rc) rc = encode_weight(enc, &maps[7 * L], h->lm_head, d, c.vocab);
+    if (!rc) rc = encode_weight(enc, &maps[7 * L], h->lm_head, d, c.vocab, kFTile);
     const bf16* planes[3] = {h->xn_hi, h->at_hi, h->ac_hi};
     const int widths[3] = {d, qd, c.ffn};
     const int rows[kPlaneClasses] = {1, 4, 8, 12, 16};
@@ -354,8 +332,8 @@ GemmArgs proj_args(ssd_handle* h, int N, int K, int n_tiles, const bf16* x_hi, c
     a.N = N;
     a.K = K;
     a.n_tiles = n_tiles;
-    a.n_chunks = (K + kStreamKC - 1) / kStreamKC;
-    a.wide = K % 64 == 0;
+    a.n_chunks = (K + kFKC - 1) / kFKC;
+    a.wide = 1;
     a.n_units = n_tiles * a.n_chunks;
     a.x_hi = x_hi;
     a.x_lo = x_lo;
@@ -375,7 +353,7 @@ GemmArgs proj_args(ssd_handle* h, int N, int K, int n_tiles, const bf16* x_hi, c
 std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
     const ssd_config& c = h->cfg;
     const int d = c.d_model, qd = c.n_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
-    const int d_tiles = d / kTileRows;
+    const int d_tiles = d / kFTile;
     std::vector<FwdOp> ops;
     FwdOp e{};
     e.type = OP_EMBED;
@@ -387,7 +365,7 @@ std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
             FwdOp q{};
             q.type = OP_QKV;
             GemmArgs& a = q.g;
-            a = proj_args(h, qd + 2 * kvd, d, (qd + 2 * kvd) / kTileRows, h->xn_hi, h->xn_lo);
+            a = proj_args(h, qd + 2 * kvd, d, (qd + 2 * kvd) / kFTile, h->xn_hi, h->xn_lo);
             a.w0 = h->wq[l]; a.w1 = h->wk[l]; a.w2 = h->wv[l];
             a.tm_w[0] = h->tmaps + tmap_weight(l, 0);
             a.tm_w[1] = h->tmaps + tmap_weight(l, 1);
@@ -424,7 +402,7 @@ std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
         if (run_m) {
             FwdOp gu{};
             gu.type = OP_SWIGLU;
-            gu.g = proj_args(h, 2 * c.ffn, d, (c.ffn + 31) / 32, h->xn_hi, h->xn_lo);
+            gu.g = proj_args(h, 2 * c.ffn, d, (c.ffn + 63) / 64, h->xn_hi, h->xn_lo);
             gu.g.w0 = h->w_gate[l]; gu.g.w1 = h->w_up[l];
             gu.g.tm_w[0] = h->tmaps + tmap_weight(l, 4);
             gu.g.tm_w[1] = h->tmaps + tmap_weight(l, 5);
@@ -445,7 +423,7 @@ std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
     }
     FwdOp lg{};
     lg.type = OP_LOGITS;
-    lg.g = proj_args(h, c.vocab, d, (c.vocab + kTileRows - 1) / kTileRows, h->xn_hi, h->xn_lo);
+    lg.g = proj_args(h, c.vocab, d, (c.vocab + kFTile - 1) / kFTile, h->xn_hi, h->xn_lo);
     lg.g.w0 = h->lm_head;
     lg.g.tm_w[0] = h->tmaps + 7 * c.n_layers;
     set_x_maps(h, lg.g, 0);
@@ -585,12 +563,14 @@ bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 int check_config(const ssd_config* c) {
     if (!c) return fail(SSD_ERR_INVALID_ARG, "config is NULL");
-    if (c->n_layers < 1 || c->d_model < 64 || c->d_model % 64)
-        return fail(SSD_ERR_INVALID_ARG, "n_layers >= 1 and d_model a positive multiple of 64 required");
+    if (c->n_layers < 1 || c->d_model < 128 || c->d_model % 128)
+        return fail(SSD_ERR_INVALID_ARG, "n_layers >= 1 and d_model a positive multiple of 128 required");
     if (c->head_dim != 64 && c->head_dim != 128)
         return fail(SSD_ERR_INVALID_ARG, "head_dim must be 64 or 128");
     if (c->n_heads < 1 || c->n_kv_heads < 1 || c->n_heads % c->n_kv_heads)
         return fail(SSD_ERR_INVALID_ARG, "n_heads must be a positive multiple of n_kv_heads");
+    if ((c->n_heads * c->head_dim) % 128 || (c->n_kv_heads * c->head_dim) % 128)
+        return fail(SSD_ERR_INVALID_ARG, "n_heads * head_dim and n_kv_heads * head_dim must be multiples of 128");
     if (c->ffn < 64 || c->ffn % 16) return fail(SSD_ERR_INVALID_ARG, "ffn must be a multiple of 16, at least 64");
     if (c->vocab < 2 || c->vocab > 32768) return fail(SSD_ERR_INVALID_ARG, "vocab must be in [2, 32768]");
     if (c->max_seq < 2 || c->max_seq > (1 << 24)) return fail(SSD_ERR_INVALID_ARG, "max_seq out of range");
@@ -695,16 +675,16 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
     h->mask.assign(2 * L, 0);
 
     // plans
-    h->p_qkv = make_plan(d, (qd + 2 * kvd) / kTileRows);
-    h->p_o = make_plan(qd, (d + kTileRows - 1) / kTileRows);
-    h->p_gu = make_plan(d, (c.ffn + 31) / 32);
-    h->p_down = make_plan(c.ffn, (d + kTileRows - 1) / kTileRows);
-    h->p_head = make_plan(d, (c.vocab + kTileRows - 1) / kTileRows);
+    // split-K slots of the forward kernel: [tile][segment <= chunks][16][128] tagged words
     size_t part = 0;
-    for (const GemmPlan* p : {&h->p_qkv, &h->p_o, &h->p_gu, &h->p_down, &h->p_head}) {
-        const int K = p == &h->p_o ? qd : (p == &h->p_down ? c.ffn : d);
-        const size_t chunks = (size_t)(K + kStreamKC - 1) / kStreamKC;
-        part = std::max(part, chunks * kMaxRows * p->n_tiles * kTileRows);
+    {
+        const int Ks[5] = {d, qd, d, c.ffn, d};
+        const int tiles[5] = {(qd + 2 * kvd) / kFTile, d / kFTile, (c.ffn + 63) / 64, d / kFTile,
+                              (c.vocab + kFTile - 1) / kFTile};
+        for (int i = 0; i < 5; ++i) {
+            const size_t chunks = (size_t)(Ks[i] + kFKC - 1) / kFKC;
+            part = std::max(part, chunks * kMaxRows * (size_t)tiles[i] * kFTile);
+        }
     }
     h->n_chunks = (c.max_seq + kAttnChunk - 1) / kAttnChunk;
     const int G = c.n_heads / c.n_kv_heads;
@@ -716,7 +696,7 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
     if ((rc = dalloc(h, &h->kc, h->kv_layer * L, &B)) || (rc = dalloc(h, &h->vc, h->kv_layer * L, &B)) ||
         (rc = dalloc(h, &h->h, (size_t)kMaxRows * d, &B)) ||
         (rc = dalloc(h, &h->xn_hi, (size_t)2 * kMaxRows * d, &B)) ||
-        (rc = dalloc(h, &h->ss, (size_t)kMaxRows * (d / kTileRows), &B)) ||
+        (rc = dalloc(h, &h->ss, (size_t)kMaxRows * (d / kFTile), &B)) ||
         (rc = dalloc(h, &h->q, (size_t)kMaxRows * qd, &B)) ||
         (rc = dalloc(h, &h->at_hi, (size_t)2 * kMaxRows * qd, &B)) ||
         (rc = dalloc(h, &h->ac_hi, (size_t)2 * kMaxRows * F, &B)) ||
@@ -773,7 +753,7 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
 
     // prefill on the tensor cores: needs the q / k / v widths in whole
     // 128-row boxes; otherwise prompts run through the decode kernel
-    h->pf_on = qd % 128 == 0 && kvd % 128 == 0;
+    h->pf_on = true;
     if (h->pf_on) {
         PrefillPlan& P = h->pf;
         P.n_layers = L;

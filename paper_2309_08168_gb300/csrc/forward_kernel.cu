@@ -14,23 +14,28 @@
 // not complete within ~2 s records an error code and the CTAs return.
 //
 // Projections (all of them: q/k/v + RoPE + KV write, output and down with the
-// residual add, gate/up with SwiGLU, lm_head): swap-AB tensor-core MMA,
-// mma.sync m16n8k16 bf16 -> fp32, 16 weight rows on the MMA's M side, the
-// activation rows as bf16 hi + lo planes on its N side (~16 mantissa bits).
-// Work unit = 64-row tile x 256-wide k chunk (32 KB of weights); each CTA
-// owns an equal contiguous range of units in tile-major order, streamed
-// through a 4-stage TMA ring.  A tile split over several CTAs is summed in
-// segment order by the CTA holding its first chunks; the others store their
-// partials tagged with the op (value and tag in one 64-bit word), so they
-// neither fence nor signal, and the finaliser polls the words themselves.
+// residual add, gate/up with SwiGLU, lm_head) run on the 5th-generation
+// tensor cores: work unit = 128-row tile x 128-wide k chunk (32 KB of
+// weights), each CTA owns an equal contiguous range of units in tile-major
+// order, streamed by TMA (128-byte swizzle) through a 4-5 stage ring; one
+// thread of the MMA warp issues tcgen05.mma kind::f16 per unit (M = 128 weight
+// rows, N = the activation rows as bf16 hi + lo planes, ~16 mantissa bits of
+// the fp32 activations) into a TMEM accumulator and releases the stage with
+// tcgen05.commit; the consumer warps read a finished tile segment from TMEM
+// (tcgen05.ld) while the next segment accumulates in the other accumulator.
+// A tile split over several CTAs is summed in segment order by the CTA
+// holding its first chunks; the others store their partials tagged with the
+// op (value and tag in one 64-bit word), so they neither fence nor signal,
+// and the finaliser polls the words themselves.
 // RMSNorm is folded in: the producer of the residual stream writes the planes
-// of h * g_next and per-64-column sums of h^2, the consumer scales row m by
+// of h * g_next and per-128-column sums of h^2, the consumer scales row m by
 // rsqrt(mean(h^2) + eps) in its epilogue (W (h g r) = r W (h g)).
 //
 // Attention: items = (KV head, absolute 128-position segment, group of 16
 // query vectors); the partial softmax of a row over a segment depends only on
-// the row and the segment, and the CTA that completes a head last combines
-// its segments in segment order.
+// the row and the segment.  After a grid barrier every CTA combines a share
+// of the (KV head, query vector) outputs over their segments in segment
+// order.
 //
 // Coherence: L1 is not coherent across SMs within one launch, so every load of
 // data another CTA wrote during this launch goes through L2 (cp.async.cg,
@@ -38,20 +43,20 @@
 //
 // Batch invariance (greedy self-speculative output must equal autoregressive
 // output bit for bit, Sec. 1 / App. G.2): row m's result depends only on row
-// m - MMA columns are independent, unit partitions and combine orders depend
-// on the shapes and the grid only, epilogues are per row, attention chunks are
-// absolute positions.
+// m - the MMA's output columns are independent (an input row is one column of
+// D whatever N is), unit partitions and combine orders depend on the shapes
+// and the grid only, epilogues are per row, attention segments are absolute
+// positions.
 #include "ssd_internal.cuh"
 
 namespace ssd {
 namespace {
 
-constexpr int KC = kStreamKC;
-constexpr int ROWB = KC * 2;  // bytes of one 64-row tile row of a unit
 constexpr unsigned long long kBarrierTimeoutNs = 2000000000ull;
-// 8 consumer warps (MMA, epilogues, attention, embedding) + 1 producer warp (TMA)
+// 8 consumer warps (epilogues, attention, embedding) + 1 producer warp (TMA)
+// + 1 MMA warp (tcgen05.mma issue, TMEM allocation)
 constexpr int kConsumers = 256;
-constexpr int kFwdThreads = kConsumers + 32;
+constexpr int kFwdThreads = kConsumers + 64;
 
 // barrier among the consumer warps only (the producer keeps streaming)
 __device__ __forceinline__ void consumer_sync() { asm volatile("bar.sync 1, 256;" ::: "memory"); }
@@ -210,13 +215,6 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const void* tmap, int x, 
         : "memory");
 }
 
-__device__ __forceinline__ void tma_load_4d(void* dst, const void* tmap, int x, int y, int z, int w, uint64_t* bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5}], [%6];"
-        ::"r"(smem_u32(dst)), "l"(tmap), "r"(x), "r"(y), "r"(z), "r"(w), "r"(smem_u32(bar))
-        : "memory");
-}
-
 __device__ __forceinline__ void tma_load_3d(void* dst, const void* tmap, int x, int y, int z, uint64_t* bar) {
     asm volatile(
         "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];"
@@ -250,18 +248,23 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
 }
 
 // ---------------------------------------------------------------------------
-// projection op
+// projection op: TMA ring -> tcgen05.mma -> TMEM -> epilogue
 // ---------------------------------------------------------------------------
-// Stage layout (1 KB aligned boxes; 128-byte swizzle: 16-byte chunk c of a
-// 128-byte smem row at address A sits at chunk c ^ ((A >> 7) & 7)).
-// wide layout (K % 64 == 0):
-//   weights: [half 2][row 32][k-box 4][64 bf16]: row r of the tile at
-//            (r >> 5) * 16 KB + (r & 31) * 512 + kbox * 128
-//   inputs : [plane 2][row R][k-box 4][64 bf16]: MMA row p = plane * R + row at
-//            p * 512 + kbox * 128 (rows past 2R only feed unused output columns)
-// narrow layout (K % 64 != 0, one copy per 64-wide k-box):
-//   weights: [k-box 4][row 64][64]: kbox * 8 KB + r * 128
-//   inputs : [k-box 4][max(2R, 8) rows][64]: kbox * XKB + p * 128
+// Work unit = a 128-row tile x 128-wide k chunk of a weight matrix (32 KB).
+// Stage layout (1 KB aligned; TMA writes the 128-byte swizzle, which is the
+// canonical K-major operand layout of tcgen05.mma: row r of a 64-wide k box
+// at r * 128 bytes, 8-row groups 1024 bytes apart):
+//   weights : k box kb (k0 + 64 kb ..) of the tile's 128 rows at kb * 16 KB
+//             (SwiGLU tiles: rows 0-63 gate, 64-127 up, of features 64 t ..)
+//   inputs  : k box kb at 32 KB + kb * XKB; rows p = plane * R + row (the R
+//             hi rows, then the R lo rows); rows 2R .. NP-1 are not written and
+//             only feed accumulator columns that nobody reads
+// One thread of the MMA warp issues, per unit, eight tcgen05.mma kind::f16
+// (bf16 x bf16 -> fp32; M = 128 weight rows, N = NP input rows, K = 16) into
+// one of two TMEM accumulators (one per tile segment, so the consumers read a
+// finished segment while the next one accumulates) and releases the stage
+// with tcgen05.commit.  The consumer warps only run the segment epilogue.
+//
 // attention: 64-position chunks per segment (one ring stage each).  Segments
 // are absolute, so a row's softmax partials do not depend on M; two chunks
 // per segment balance ~150 CTAs well at LLaMA-2 KV-head counts and contexts
@@ -271,7 +274,7 @@ constexpr int kAttnSegChunks = 2;
 // Attention unit in a stage: K rows of the 64-position chunk at 0 (dims 0-63,
 // then 64-127 at 8 KB), V rows at 16 KB; position t, 16-byte chunk c of a
 // 64-dim box at box + t * 128 + ((c ^ (t & 7)) << 4).
-// After the ring: the consumers' scratch - split-K reduction buffers of a
+// After the ring: the consumers' scratch - the finished segment of a
 // projection, or (same bytes: one op at a time) q / scores of attention.
 // index of the input-plane tensor map of R rows
 __host__ __device__ constexpr int plane_cls(int R) {
@@ -280,98 +283,124 @@ __host__ __device__ constexpr int plane_cls(int R) {
 
 template <int R>
 struct GemmSmem {
-    static constexpr int NT = (2 * R + 7) / 8;   // n8 MMA tiles: 1 | 2 | 4
-    static constexpr int XR = NT * 8;            // input rows the MMA reads
-    static constexpr int WB = kTileRows * ROWB;  // 32 KB
-    static constexpr int XKB = XR * 128;         // narrow layout: input bytes per k-box
-    static constexpr int XB = XR * ROWB;         // = 4 * XKB
-    static constexpr int STAGE = WB + XB;
-    static constexpr int RC = NT * 8;
+    static constexpr int NP = R <= 8 ? 16 : 32;     // MMA N: input rows (hi + lo), padded
+    static constexpr int WB = kFTile * kFKC * 2;    // 32 KB of weights per unit
+    static constexpr int XKB = NP * 128;            // input bytes per 64-wide k box
+    static constexpr int STAGE = WB + 2 * XKB;
+    static constexpr int S = R <= 8 ? 5 : 4;        // ring depth
     static constexpr int VG = 16;  // attention: query vectors per item (one MMA M / N tile)
-    static constexpr int S = 4;  // ring depth (5 or 6 stages, where they fit, measured no faster)
-    static constexpr int RED = S * STAGE;                // [64][RC] floats
-    static constexpr int YS = RED + kTileRows * RC * 4;  // [64][16] floats
+    static constexpr int YS = S * STAGE;            // [128][16] floats: the finished segment
     // attention scratch: q hi / lo (fp16, rows padded by 16 bytes), scores
     // (fp32), P hi / lo (fp16, padded rows)
     static constexpr int QST = 128 + 8, PST = kAttnSegChunks * kAttnChunk + 8;  // halves per row
-    static constexpr int ATT = RED;
+    static constexpr int ATT = S * STAGE;
     static constexpr int ATT_SC = ATT + 2 * VG * QST * 2;
     static constexpr int ATT_P = ATT_SC + VG * kAttnSegChunks * kAttnChunk * 4;
-    static constexpr int SCRATCH_GEMM = kTileRows * RC * 4 + kTileRows * 16 * 4;
+    static constexpr int SCRATCH_GEMM = kFTile * 16 * 4;
     static constexpr int SCRATCH_ATT = ATT_P + 2 * VG * PST * 2 - ATT;
     static constexpr size_t BYTES =
-        1024 + (size_t)RED + (SCRATCH_GEMM > SCRATCH_ATT ? SCRATCH_GEMM : SCRATCH_ATT);
+        1024 + (size_t)S * STAGE + (SCRATCH_GEMM > SCRATCH_ATT ? SCRATCH_GEMM : SCRATCH_ATT);
+    static_assert(STAGE >= 2 * kAttnChunk * 128 * 2, "a stage holds the K and V rows of one 64-position chunk");
 };
 
-// byte offset of 16-byte chunk c (0..7) of k-box kb in row r of the weights,
-// or row p of the inputs (the swizzle XOR follows the address)
-__device__ __forceinline__ int w_off(bool wide, int r, int kb, int c) {
-    if (wide) {
-        const int a = (r >> 5) * 16384 + (r & 31) * 512 + kb * 128;
-        return a + ((c ^ ((a >> 7) & 7)) << 4);
-    }
-    const int a = kb * 8192 + r * 128;
-    return a + ((c ^ (r & 7)) << 4);
+// ---------------------------------------------------------------------------
+// tcgen05 helpers
+// ---------------------------------------------------------------------------
+constexpr int kTmemCols = 64;  // two accumulators of up to 32 fp32 columns
+
+// shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart; the start address may sit 32 / 64 / 96 bytes into a
+// swizzle row (k steps of 16 bf16)
+__device__ __forceinline__ uint64_t umma_desc(uint32_t saddr) {
+    uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address
+    d |= (uint64_t)1 << 16;                           // leading byte offset (unused with this swizzle)
+    d |= (uint64_t)(1024 >> 4) << 32;                 // stride byte offset
+    d |= (uint64_t)1 << 46;                           // descriptor version
+    d |= (uint64_t)2 << 61;                           // 128-byte swizzle
+    return d;
 }
-template <int R>
-__device__ __forceinline__ int x_off(bool wide, int p, int kb, int c) {
-    if (wide) {
-        const int a = p * 512 + kb * 128;
-        return a + ((c ^ ((a >> 7) & 7)) << 4);
-    }
-    const int a = kb * GemmSmem<R>::XKB + p * 128;
-    return a + ((c ^ (p & 7)) << 4);
+// instruction descriptor: kind::f16, A = B = bf16, D = fp32, both K-major,
+// M = 128, N = np
+__host__ __device__ constexpr uint32_t umma_idesc(int np) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(np >> 3) << 17) | ((uint32_t)(kFTile >> 4) << 24);
+}
+__device__ __forceinline__ void umma(uint32_t tmem_d, uint64_t ad, uint64_t bd, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n"
+        ::"r"(tmem_d), "l"(ad), "l"(bd), "r"(idesc), "r"(acc)
+        : "memory");
+}
+// the mbarrier completes once every tcgen05 op this thread issued so far is done
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// NP consecutive fp32 columns of this thread's TMEM lane
+template <int NP>
+__device__ __forceinline__ void tmem_ld(uint32_t taddr, float (&v)[NP]);
+template <>
+__device__ __forceinline__ void tmem_ld<16>(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+template <>
+__device__ __forceinline__ void tmem_ld<32>(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// Sources of a 64-row tile as two 32-row halves: rows r0.. of matrix s0, then
-// rows r1.. of matrix s1 (0, 1, 2 = w0, w1, w2).  Halves come from two places
-// for the RoPE pairs of q / k (rotation partners j and j + head_dim/2) and for
-// gate + up.
-struct Halves {
-    int s0, r0, s1, r1;
+// Weight rows of tile t: one 128-row box (matrix s0 from row r0), or for
+// SwiGLU two 64-row boxes (the gate and the up rows of features 64 t ..).
+// The q / k / v widths are whole tiles, so a q / k tile is 128 / head_dim
+// whole heads in natural order and holds every RoPE pair (j, j + hd / 2).
+struct TileSrc {
+    int s0, r0, s1, r1;  // s1 < 0: one box
 };
-__device__ __forceinline__ Halves tile_halves(const GemmArgs& a, int epi, int tile) {
-    if (epi == EPI_LOGITS || epi == EPI_RESID) return {0, tile * kTileRows, 0, tile * kTileRows + 32};
-    if (epi == EPI_SWIGLU) return {0, tile * 32, 1, tile * 32};  // gate rows, up rows
-    const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
-    const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
-    if (tile < q_tiles + k_tiles) {
-        const bool is_q = tile < q_tiles;
-        const int tt = is_q ? tile : tile - q_tiles;
-        const int head = tt / per_head, j0 = (tt % per_head) * 32;
-        const int sm = is_q ? 0 : 1;
-        return {sm, head * hd + j0, sm, head * hd + half + j0};
+__device__ __forceinline__ TileSrc tile_src(const GemmArgs& a, int epi, int tile) {
+    if (epi == EPI_SWIGLU) return {0, tile * 64, 1, tile * 64};
+    if (epi == EPI_QKV) {
+        const int qt = a.n_heads * a.head_dim / kFTile, kt = a.n_kv_heads * a.head_dim / kFTile;
+        if (tile < qt) return {0, tile * kFTile, -1, 0};
+        if (tile < qt + kt) return {1, (tile - qt) * kFTile, -1, 0};
+        return {2, (tile - qt - kt) * kFTile, -1, 0};
     }
-    const int r = (tile - q_tiles - k_tiles) * kTileRows;
-    return {2, r, 2, r + 32};
-}
-
-__device__ __forceinline__ int unit_kboxes(const GemmArgs& a, int u) {
-    const int k0 = (u % a.n_chunks) * KC;
-    return min(4, (a.K - k0 + 63) / 64);
+    return {0, tile * kFTile, -1, 0};
 }
 
 // weights of unit u into a stage (one thread): expect_tx without arriving.
-// Bytes are always a full 64 x 256 tile (out-of-range rows / columns are
-// delivered as zeros and counted).
+// Always a full 128 x 128 tile of bytes (rows / columns out of range are
+// delivered as zeros and counted).  Every x used here is a multiple of 64
+// elements (128 bytes), so the 16-byte rule for x * element size holds.
 template <int R>
 __device__ __forceinline__ void tma_weights(const GemmArgs& a, int epi, int u, unsigned char* st, uint64_t* bar) {
-    const int tile = u / a.n_chunks, k0 = (u - tile * a.n_chunks) * KC;
-    const Halves hv = tile_halves(a, epi, tile);
-    const void* m0 = a.tm_w[hv.s0];
-    const void* m1 = a.tm_w[hv.s1];
-    const int r0 = hv.r0, r1 = hv.r1;
-    if (a.wide) {
-        mbar_expect_tx(bar, 32768u);
-        tma_load_3d(st, m0, 0, k0 >> 6, r0, bar);
-        tma_load_3d(st + 16384, m1, 0, k0 >> 6, r1, bar);
-    } else {
-        const int nkb = unit_kboxes(a, u);
-        mbar_expect_tx(bar, (unsigned)nkb * 8192u);
-        for (int kb = 0; kb < nkb; ++kb) {
-            tma_load_2d(st + kb * 8192, m0, k0 + kb * 64, r0, bar);
-            tma_load_2d(st + kb * 8192 + 4096, m1, k0 + kb * 64, r1, bar);
-        }
+    const int tile = u / a.n_chunks, k0 = (u - tile * a.n_chunks) * kFKC;
+    const TileSrc ts = tile_src(a, epi, tile);
+    mbar_expect_tx(bar, (unsigned)GemmSmem<R>::WB);
+#pragma unroll
+    for (int kb = 0; kb < 2; ++kb) {
+        tma_load_2d(st + kb * 16384, a.tm_w[ts.s0], k0 + kb * 64, ts.r0, bar);
+        if (ts.s1 >= 0) tma_load_2d(st + kb * 16384 + 8192, a.tm_w[ts.s1], k0 + kb * 64, ts.r1, bar);
     }
 }
 
@@ -379,28 +408,42 @@ __device__ __forceinline__ void tma_weights(const GemmArgs& a, int epi, int u, u
 template <int R>
 __device__ __forceinline__ void tma_inputs(const GemmArgs& a, int u, unsigned char* st, uint64_t* bar) {
     using L = GemmSmem<R>;
-    const int k0 = (u % a.n_chunks) * KC;
+    const int k0 = (u % a.n_chunks) * kFKC;
     const int cls = plane_cls(R);
-    unsigned char* xs = st + L::WB;
-    if (a.wide) {
-        mbar_arrive_expect_tx(bar, 4u * 2u * (unsigned)R * 128u);
-        tma_load_4d(xs, a.tm_x[cls], 0, k0 >> 6, 0, 0, bar);
-    } else {
-        const int nkb = unit_kboxes(a, u);
-        mbar_arrive_expect_tx(bar, (unsigned)nkb * 2u * (unsigned)R * 128u);
-        for (int kb = 0; kb < nkb; ++kb) tma_load_3d(xs + kb * L::XKB, a.tm_x[cls], k0 + kb * 64, 0, 0, bar);
-    }
+    mbar_arrive_expect_tx(bar, 2u * 2u * (unsigned)R * 128u);
+#pragma unroll
+    for (int kb = 0; kb < 2; ++kb) tma_load_3d(st + L::WB + kb * L::XKB, a.tm_x[cls], k0 + kb * 64, 0, 0, bar);
 }
 
-// Pipeline state of the CTA, carried across ops.  Producer: pphase bit s =
-// parity of the next "empty" completion of stage s to wait for.  Consumers:
-// cphase bit s = parity of the next "full" completion.
+// Pipeline state, carried across ops; every thread keeps its own copy and
+// flips the bits of the waits it takes part in (or, for ring positions whose
+// waits another role took, the same bits arithmetically).
+//   pphase bit s : parity of the next "empty" completion of stage s (producer)
+//   cphase bit s : parity of the next "full" completion of stage s (MMA thread
+//                  in projections, consumers in attention)
+//   afull bit b  : parity of the next completion of accumulator b (consumers)
+//   aempty bit b : parity of the next release of accumulator b (MMA thread)
+//   ab           : accumulator of the next tile segment
 struct Pipe {
-    uint64_t* full;   // [stages] TMA completion (count 1: the producer's arrive)
-    uint64_t* empty;  // [stages] stage released (count 8: one arrive per consumer warp)
+    uint64_t* full;     // [stages] TMA completion (count 1: the producer's arrive)
+    uint64_t* empty;    // [stages] stage released (count 1: tcgen05.commit, or consumer thread 0)
+    uint64_t* acc_full;   // [2] accumulator complete (tcgen05.commit)
+    uint64_t* acc_empty;  // [2] accumulator read by the consumers (thread 0)
+    uint32_t tmem;      // TMEM base address (two accumulators of kTmemCols / 2 columns)
     unsigned pphase;
     unsigned cphase;
+    unsigned afull;
+    unsigned aempty;
+    int ab;
 };
+
+// flips the full-barrier parity bits of n consecutive ring positions from 0
+template <int S>
+__device__ __forceinline__ void advance_full(Pipe& pp, int n) {
+#pragma unroll
+    for (int s = 0; s < S; ++s)
+        if (((n / S) + (s < n % S ? 1 : 0)) & 1) pp.cphase ^= 1u << s;
+}
 
 // Producer: requests the weights of this CTA's first S units of a projection
 // before the grid barrier (they do not depend on the previous op).
@@ -423,21 +466,22 @@ __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, P
     return ok;
 }
 
-// Returns false if a TMA wait timed out (error recorded).  The producer warp
-// (one elected thread) streams this CTA's units through the S stages; the 8
-// consumer warps compute and release each stage with one arrival per warp.
+// Returns false if a wait timed out (error recorded).  Three roles:
+//   producer (one thread of warp 8) streams this CTA's units through the ring;
+//   MMA issuer (one thread of warp 9) runs tcgen05.mma per unit into the
+//     accumulator of the unit's tile segment;
+//   consumers (warps 0-7), per finished segment: TMEM -> hi + lo summed ->
+//     split-K exchange -> epilogue.
 // ut: nullptr, or [64][4] timestamps of this CTA's first units (producer
-// issue, consumer data ready, MMA done, flush done); ct: nullptr, or this
-// CTA's op stamps (FwdParams::trace) - profiling aids.
+// issue, MMAs issued, 0, segment flush done); ct: nullptr, or this CTA's op
+// stamps (FwdParams::trace) - profiling aids.
 template <int R>
 __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefetched, unsigned char* smem,
                         float* r_s, Pipe& pp, unsigned tag, int* err, unsigned long long* ut,
                         unsigned long long* ct) {
     using L = GemmSmem<R>;
-    constexpr int NT = L::NT, RC = L::RC;
-    constexpr int S = L::S;
-    float* red = reinterpret_cast<float*>(smem + L::RED);  // [64][RC]
-    float* ys = reinterpret_cast<float*>(smem + L::YS);    // [64][16]
+    constexpr int S = L::S, NP = L::NP;
+    float* ys = reinterpret_cast<float*>(smem + L::YS);  // [128][16]
     bool ok = true;
 
     const long long U = a.n_units, G = op_ctas(U);
@@ -445,9 +489,10 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
     int u_begin, n_my;
     my_units(U, &u_begin, &n_my);
 
-    if (threadIdx.x >= kConsumers) {  // producer warp: one elected thread drives the ring
+    if (threadIdx.x >= kConsumers && threadIdx.x < kConsumers + 32) {  // producer warp
         if (threadIdx.x != kConsumers) return true;
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        asm volatile("fence.proxy.async.global;" ::: "memory");  // inputs written by the previous op
         for (int i = 0; i < n_my; ++i) {
             const int s = i % S;
             unsigned char* st = smem + s * L::STAGE;
@@ -458,6 +503,41 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
                 tma_weights<R>(a, epi, u_begin + i, st, pp.full + s);
             }
             tma_inputs<R>(a, u_begin + i, st, pp.full + s);
+        }
+        return true;
+    }
+
+    if (threadIdx.x >= kConsumers + 32) {  // MMA warp: one elected thread issues
+        if (threadIdx.x != kConsumers + 32) return true;
+        constexpr uint32_t idesc = umma_idesc(NP);
+        for (int i = 0; i < n_my; ++i) {
+            const int u = u_begin + i;
+            const int chunk = u % a.n_chunks;
+            const bool first = i == 0 || chunk == 0;
+            const bool last = i == n_my - 1 || chunk == a.n_chunks - 1;
+            const int ab = pp.ab;
+            if (first) {  // the consumers have read this accumulator's previous segment
+                if (!mbar_wait(pp.acc_empty + ab, (pp.aempty >> ab) & 1u, err)) return false;
+                pp.aempty ^= 1u << ab;
+            }
+            const int s = i % S;
+            if (!mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err)) return false;
+            pp.cphase ^= 1u << s;
+            tc_fence_after();
+            const uint32_t st = smem_u32(smem + s * L::STAGE);
+            const uint32_t d = pp.tmem + (uint32_t)(ab * (kTmemCols / 2));
+#pragma unroll
+            for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma(d, umma_desc(st + kb * 16384 + ks * 32), umma_desc(st + L::WB + kb * L::XKB + ks * 32),
+                         idesc, (first && kb == 0 && ks == 0) ? 0u : 1u);
+            umma_commit(pp.empty + s);  // the stage is free once these MMAs have read it
+            if (ut && i < 64) ut[i * 4 + 1] = globaltimer();
+            if (last) {
+                umma_commit(pp.acc_full + ab);
+                pp.ab ^= 1;
+            }
         }
         return true;
     }
@@ -475,137 +555,66 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         }
         if (lane == 0) r_s[m] = r;
     }
-
-    const int rg = warp & 3, kh = warp >> 2;
-    const int g = lane >> 2, tig = lane & 3;
-    const int r0 = rg * 16 + g;
-    // two accumulator sets (k32 blocks kh, kh+4 | kh+2, kh+6) halve the MMA chain
-    float acc[NT][4], acc2[NT][4];
-#pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
-        acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = acc2[nt][0] = acc2[nt][1] = acc2[nt][2] =
-            acc2[nt][3] = 0.f;
+    // the MMA thread took the full-barrier waits of these ring positions
+    advance_full<S>(pp, n_my);
 
     for (int i = 0; i < n_my; ++i) {
         const int u = u_begin + i;
         const int tile = u / a.n_chunks, chunk = u - tile * a.n_chunks;
-        const int kc_eff = min(KC, a.K - chunk * KC);
-        const int s = i % S;
-        const unsigned char* w_s = smem + s * L::STAGE;
-        const unsigned char* x_s = w_s + L::WB;
-        // a failed wait leaves garbage in the stage: carry on (every consumer
-        // must reach every consumer barrier), the error is reported
-        ok = mbar_wait(pp.full + s, (pp.cphase >> s) & 1u, err) && ok;
-        pp.cphase ^= 1u << s;
-        if (threadIdx.x == 0) {
-            if (ut && i < 64) ut[i * 4 + 1] = globaltimer();
-            if (ct && i == 0) ct[1] = globaltimer();
-        }
-
-        // A: weight rows r0, r0 + 8; B: input rows nt*8 + g.  Both operands use
-        // the same chunk -> logical-k mapping, so the product is unchanged;
-        // columns past K are zero-filled by TMA in both operands.
-        const int nb = (kc_eff + 31) >> 5;
-        const bool wide = a.wide != 0;
-        auto block = [&](int kb, float (&ac)[NT][4]) {
-            // k32 block kb = 16-byte chunks 4*(kb&1) .. +3 of k-box kb/2; thread tig takes chunk 4*(kb&1) + tig
-            const int kbx = kb >> 1, c = 4 * (kb & 1) + tig;
-            const uint4 wa = *reinterpret_cast<const uint4*>(w_s + w_off(wide, r0, kbx, c));
-            const uint4 wb = *reinterpret_cast<const uint4*>(w_s + w_off(wide, r0 + 8, kbx, c));
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                const uint4 xv = *reinterpret_cast<const uint4*>(x_s + x_off<R>(wide, nt * 8 + g, kbx, c));
-                mma_bf16_16816(ac[nt], wa.x, wb.x, wa.y, wb.y, xv.x, xv.y);
-                mma_bf16_16816(ac[nt], wa.z, wb.z, wa.w, wb.w, xv.z, xv.w);
-            }
-        };
-        for (int kb = kh; kb < nb; kb += 4) {
-            block(kb, acc);
-            if (kb + 2 < nb) block(kb + 2, acc2);
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(pp.empty + s);  // this warp is done with the stage
-        if (threadIdx.x == 0) {
-            if (ut && i < 64) ut[i * 4 + 2] = globaltimer();
-            if (ct && i == n_my - 1) {
-                ct[2] = globaltimer();
-                ct[6] = (unsigned long long)n_my;
-            }
-        }
-
+        if (threadIdx.x == 0 && ct && i == n_my - 1) ct[6] = (unsigned long long)n_my;
         if (!(i == n_my - 1 || chunk == a.n_chunks - 1)) continue;
 
-        // this CTA's segment of the tile is complete: accumulator sets, then
-        // k-interleaves, then hi + lo
+        // this CTA's segment of the tile is complete: its accumulator holds
+        // W x_hi in columns 0..R-1 and W x_lo in columns R..2R-1
+        const int ab = pp.ab;
+        ok = mbar_wait(pp.acc_full + ab, (pp.afull >> ab) & 1u, err) && ok;
+        pp.afull ^= 1u << ab;
+        pp.ab ^= 1;
+        tc_fence_after();
+        if (threadIdx.x == 0 && ct) ct[2] = globaltimer();
+        if (warp < 4) {  // warp w reads TMEM lanes (tile rows) 32w .. 32w + 31
+            float v[NP];
+            tmem_ld<NP>(pp.tmem + (uint32_t)(ab * (kTmemCols / 2)) + ((uint32_t)(warp * 32) << 16), v);
+            const int r = warp * 32 + lane;
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                acc[nt][e] = acc[nt][e] + acc2[nt][e];
-                acc2[nt][e] = 0.f;
-            }
-        if (kh == 1) {
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                const int c = nt * 8 + 2 * tig;
-                red[r0 * RC + c] = acc[nt][0];
-                red[r0 * RC + c + 1] = acc[nt][1];
-                red[(r0 + 8) * RC + c] = acc[nt][2];
-                red[(r0 + 8) * RC + c + 1] = acc[nt][3];
-            }
+            for (int m = 0; m < R; ++m) ys[r * 16 + m] = v[m] + v[R + m];
         }
+        tc_fence_before();
         consumer_sync();
-        if (kh == 0) {
-#pragma unroll
-            for (int nt = 0; nt < NT; ++nt) {
-                const int c = nt * 8 + 2 * tig;
-                red[r0 * RC + c] = acc[nt][0] + red[r0 * RC + c];
-                red[r0 * RC + c + 1] = acc[nt][1] + red[r0 * RC + c + 1];
-                red[(r0 + 8) * RC + c] = acc[nt][2] + red[(r0 + 8) * RC + c];
-                red[(r0 + 8) * RC + c + 1] = acc[nt][3] + red[(r0 + 8) * RC + c + 1];
-            }
-        }
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
-        consumer_sync();
+        if (threadIdx.x == 0) mbar_arrive(pp.acc_empty + ab);  // the accumulator may be refilled
 
         // split-K: the CTA holding the tile's first chunks (its segment ends
         // last, at the end of that CTA's range) finalises; the others store
-        // their partial (hi + lo plane columns summed) and move on.  Each value
-        // travels with the op's tag in one 64-bit word, so the finaliser needs
-        // no flag and no fence: it reads each word until the tag is this op's.
-        // The sum is in segment order.
+        // their partial and move on.  Each value travels with the op's tag in
+        // one 64-bit word, so the finaliser needs no flag and no fence: it
+        // reads each word until the tag is this op's.  The sum is in segment
+        // order.
         const long long u_first = (long long)tile * a.n_chunks;
         const int seg0 = unit_owner(u_first, U, G);
         const int nseg = unit_owner(u_first + a.n_chunks - 1, U, G) - seg0 + 1;
-        constexpr size_t kSlot = (size_t)kMaxRows * kTileRows;
+        constexpr size_t kSlot = (size_t)kMaxRows * kFTile;
         unsigned long long* slots =
             reinterpret_cast<unsigned long long*>(a.partial) + (size_t)tile * a.n_chunks * kSlot;
         if (nseg > 1 && b != seg0) {
             unsigned long long* mine = slots + (size_t)(b - seg0) * kSlot;
-            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
-                const int m = idx / kTileRows, r = idx - m * kTileRows;
-                st_relaxed_u64(mine + m * kTileRows + r, tagged(tag, red[r * RC + m] + red[r * RC + R + m]));
+            for (int idx = threadIdx.x; idx < M * kFTile; idx += kGemmThreads) {
+                const int m = idx / kFTile, r = idx - m * kFTile;
+                st_relaxed_u64(mine + m * kFTile + r, tagged(tag, ys[r * 16 + m]));
             }
-            consumer_sync();  // red is free for the next segment
+            consumer_sync();  // ys is free for the next segment
             continue;
         }
-        for (int idx = threadIdx.x; idx < kTileRows * M; idx += kGemmThreads) {
-            const int m = idx / kTileRows, r = idx - m * kTileRows;
-            ys[r * 16 + m] = red[r * RC + m] + red[r * RC + R + m];
-        }
-        consumer_sync();
 
         // RESID: this tile's residual h (written by earlier ops: L2), loaded
         // before waiting for the other segments so its latency overlaps it
-        constexpr int HJ = kMaxRows * kTileRows / kGemmThreads;
+        constexpr int HJ = kMaxRows * kFTile / kGemmThreads;
         float hpre[HJ], gpre[HJ];
         if (epi == EPI_RESID) {
 #pragma unroll
             for (int j = 0; j < HJ; ++j) {
                 const int idx = threadIdx.x + j * kGemmThreads;
-                const int m = idx / kTileRows, n = tile * kTileRows + (idx - m * kTileRows);
-                const bool in = idx < M * kTileRows && n < a.N;
+                const int m = idx / kFTile, n = tile * kFTile + (idx - m * kFTile);
+                const bool in = idx < M * kFTile && n < a.N;
                 hpre[j] = in ? __ldcg(a.out_f32 + (size_t)m * a.ldo + n) : 0.f;
                 gpre[j] = (in && a.g_next) ? __bfloat162float(a.g_next[n]) : 0.f;
             }
@@ -613,9 +622,9 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 
         if (nseg > 1) {
             // the other segments come from later CTAs, which never wait on this one
-            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
-                const int m = idx / kTileRows, r = idx - m * kTileRows;
-                const unsigned long long* p = slots + m * kTileRows + r;
+            for (int idx = threadIdx.x; idx < M * kFTile; idx += kGemmThreads) {
+                const int m = idx / kFTile, r = idx - m * kFTile;
+                const unsigned long long* p = slots + m * kFTile + r;
                 float sum = ys[r * 16 + m];
                 for (int sg0 = 1; sg0 < nseg; sg0 += 4) {
                     unsigned long long w[4];
@@ -637,18 +646,18 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 
         // epilogue of the finished tile (row m scaled by its RMSNorm factor)
         if (epi == EPI_LOGITS) {
-            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
-                const int m = idx / kTileRows, r = idx - m * kTileRows;
-                const int n = tile * kTileRows + r;
+            for (int idx = threadIdx.x; idx < M * kFTile; idx += kGemmThreads) {
+                const int m = idx / kFTile, r = idx - m * kFTile;
+                const int n = tile * kFTile + r;
                 if (n < a.N) a.out_f32[(size_t)m * a.ldo + n] = ys[r * 16 + m] * r_s[m];
             }
         } else if (epi == EPI_RESID) {
 #pragma unroll
             for (int j = 0; j < HJ; ++j) {
                 const int idx = threadIdx.x + j * kGemmThreads;
-                if (idx >= M * kTileRows) break;
-                const int m = idx / kTileRows, r = idx - m * kTileRows;
-                const int n = tile * kTileRows + r;
+                if (idx >= M * kFTile) break;
+                const int m = idx / kFTile, r = idx - m * kFTile;
+                const int n = tile * kFTile + r;
                 float hv = 0.f;
                 if (n < a.N) {
                     float* o = a.out_f32 + (size_t)m * a.ldo + n;
@@ -666,32 +675,34 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
             if (a.g_next) {
                 consumer_sync();
                 for (int m = warp; m < M; m += kGemmThreads / 32) {
-                    const float sq = warp_sum(ys[lane * 16 + m] + ys[(lane + 32) * 16 + m]);
+                    const float sq = warp_sum((ys[lane * 16 + m] + ys[(lane + 32) * 16 + m]) +
+                                              (ys[(lane + 64) * 16 + m] + ys[(lane + 96) * 16 + m]));
                     if (lane == 0) a.ss_out[m * a.n_tiles + tile] = sq;
                 }
             }
         } else if (epi == EPI_SWIGLU) {
-            for (int idx = threadIdx.x; idx < M * 32; idx += kGemmThreads) {
-                const int m = idx >> 5, r = idx & 31;
-                const int i2 = tile * 32 + r;
+            for (int idx = threadIdx.x; idx < M * 64; idx += kGemmThreads) {
+                const int m = idx >> 6, r = idx & 63;
+                const int i2 = tile * 64 + r;
                 if (i2 >= a.ffn) continue;
-                const float gt = ys[r * 16 + m] * r_s[m], up = ys[(r + 32) * 16 + m] * r_s[m];
+                const float gt = ys[r * 16 + m] * r_s[m], up = ys[(r + 64) * 16 + m] * r_s[m];
                 const float act = gt / (1.f + expf(-gt)) * up;
                 const bf16 ah = __float2bfloat16_rn(act);
                 a.xo_hi[(size_t)m * a.ffn + i2] = ah;
                 a.xo_lo[(size_t)m * a.ffn + i2] = __float2bfloat16_rn(act - __bfloat162float(ah));
             }
         } else {  // EPI_QKV
-            const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
-            const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
-            if (tile < q_tiles + k_tiles) {
-                const bool is_q = tile < q_tiles;
-                const int tt = is_q ? tile : tile - q_tiles;
-                const int head = tt / per_head, j0 = (tt % per_head) * 32;
-                for (int idx = threadIdx.x; idx < M * 32; idx += kGemmThreads) {
-                    const int m = idx >> 5, r = idx & 31;
-                    const int ii = j0 + r, pos = pos0 + m;
-                    const float x1 = ys[r * 16 + m] * r_s[m], x2 = ys[(r + 32) * 16 + m] * r_s[m];
+            const int hd = a.head_dim, half = hd >> 1;
+            const int qt = a.n_heads * hd / kFTile, kt = a.n_kv_heads * hd / kFTile;
+            if (tile < qt + kt) {
+                const bool is_q = tile < qt;
+                const int tt = is_q ? tile : tile - qt;
+                for (int idx = threadIdx.x; idx < M * 64; idx += kGemmThreads) {
+                    const int m = idx >> 6, pr = idx & 63;  // rotation pair pr of the tile
+                    const int hl = pr / half, ii = pr - hl * half;
+                    const int r1 = hl * hd + ii, r2 = r1 + half;
+                    const int head = tt * (kFTile / hd) + hl, pos = pos0 + m;
+                    const float x1 = ys[r1 * 16 + m] * r_s[m], x2 = ys[r2 * 16 + m] * r_s[m];
                     const float2 cs = a.rope[(size_t)pos * half + ii];
                     const float y1 = x1 * cs.x - x2 * cs.y;
                     const float y2 = x2 * cs.x + x1 * cs.y;
@@ -706,17 +717,17 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
                     }
                 }
             } else {
-                const int vt = tile - q_tiles - k_tiles;
-                for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
-                    const int m = idx / kTileRows, r = idx - m * kTileRows;
-                    const int f = vt * kTileRows + r;
+                const int vt = tile - qt - kt;
+                for (int idx = threadIdx.x; idx < M * kFTile; idx += kGemmThreads) {
+                    const int m = idx / kFTile, r = idx - m * kFTile;
+                    const int f = vt * kFTile + r;
                     const int head = f / hd, e = f - head * hd;
                     a.v_cache[((size_t)head * a.max_seq + pos0 + m) * hd + e] =
                         __float2half_rn(ys[r * 16 + m] * r_s[m]);
                 }
             }
         }
-        consumer_sync();  // ys / red are reused by the next segment
+        consumer_sync();  // ys is reused by the next segment
         if (ut && i < 64 && threadIdx.x == 0) ut[i * 4 + 3] = globaltimer();
     }
     consumer_sync();
@@ -809,6 +820,17 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
     const int G = a.n_heads / a.n_kv_heads, NV = G * M;
     const AttnRange ar = attn_range(a, M, pos0);
 
+    if (threadIdx.x >= kConsumers + 32) {  // MMA warp: only keeps its copy of the ring parities
+        if (threadIdx.x == kConsumers + 32) {
+            int n = 0;
+            for (int it = ar.i_begin; it < ar.i_end; ++it) {
+                const int sg = (it / ar.n_vg) % ar.n_seg;
+                n += min(SC, ar.n_ch - sg * SC);
+            }
+            advance_full<S>(pp, n);
+        }
+        return true;
+    }
     if (threadIdx.x >= kConsumers) {  // producer warp: one elected thread requests K / V
         if (threadIdx.x != kConsumers) return true;
         // K / V rows of this forward were stored by other CTAs (generic proxy)
@@ -981,8 +1003,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
         }
         consumer_sync();  // q / scores / weights are free for the next item
         stamp(it, 6);
-        __syncwarp();
-        if (lane == 0)
+        if (tid == 0)
             for (int j = 0; j < n_u; ++j) mbar_arrive(pp.empty + (i + j) % S);  // the stages are free
         i += n_u;
     }
@@ -1049,7 +1070,7 @@ __device__ void attn_combine(const AttnArgs& a, int M, int pos0) {
 // ---------------------------------------------------------------------------
 __device__ void embed_op(const FwdParams& p, int pos0) {
     if (threadIdx.x >= kConsumers) return;
-    const int d = p.d, n_tiles = d / 64;
+    const int d = p.d, n_tiles = d / kFTile;  // sums of squares per 128 columns
     const int lane = threadIdx.x & 31;
     const int gw = blockIdx.x * (kGemmThreads / 32) + (threadIdx.x >> 5);
     const int nw = gridDim.x * (kGemmThreads / 32);
@@ -1063,8 +1084,8 @@ __device__ void embed_op(const FwdParams& p, int pos0) {
         const bf16* row = p.embed + (size_t)tok * d;
         float sq = 0.f;
 #pragma unroll
-        for (int j = 0; j < 2; ++j) {
-            const int i = t * 64 + j * 32 + lane;
+        for (int j = 0; j < kFTile / 32; ++j) {
+            const int i = t * kFTile + j * 32 + lane;
             const float v = __bfloat162float(row[i]);
             p.h[(size_t)m * d + i] = v;
             const float z = v * __bfloat162float(p.g0[i]);
@@ -1103,12 +1124,16 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
     __shared__ float r_s[kMaxRows];
     __shared__ int s_pos0, s_fail, s_skip;
     __shared__ unsigned s_seq;
+    __shared__ uint32_t s_tmem;
     constexpr int S = GemmSmem<R>::S;
-    __shared__ __align__(8) uint64_t full[S];   // TMA completion per stage
-    __shared__ __align__(8) uint64_t empty[S];  // stage released by the 8 consumer warps
-    __shared__ FwdOp s_op[2];                   // current and next op's arguments
+    __shared__ __align__(8) uint64_t full[S];       // TMA completion per stage
+    __shared__ __align__(8) uint64_t empty[S];      // stage released (tcgen05.commit, or one consumer thread)
+    __shared__ __align__(8) uint64_t acc_full[2];   // TMEM accumulator complete (tcgen05.commit)
+    __shared__ __align__(8) uint64_t acc_empty[2];  // TMEM accumulator read by the consumers
+    __shared__ FwdOp s_op[2];                       // current and next op's arguments
     // 128-byte TMA swizzle needs 1 KB aligned boxes
     unsigned char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    const bool mma_warp = threadIdx.x >= kConsumers + 32;
     if (threadIdx.x == 0) {
         int pos0;
         if (p.src == SRC_TOKENS) pos0 = p.pos0_arg;
@@ -1121,7 +1146,11 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         s_seq = *(volatile unsigned*)p.seq;  // this forward's number (advanced by CTA 0 below)
         for (int st = 0; st < S; ++st) {
             mbar_init(full + st, 1);
-            mbar_init(empty + st, kConsumers / 32);
+            mbar_init(empty + st, 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(acc_full + b, 1);
+            mbar_init(acc_empty + b, 1);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -1129,9 +1158,21 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
     }
     __syncthreads();
     if (s_skip) return;
-    // every stage starts empty: each consumer warp releases it once
-    if (threadIdx.x < kConsumers && (threadIdx.x & 31) == 0)
+    if (mma_warp) {  // TMEM for the two projection accumulators (freed at the end)
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&s_tmem)),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    // every stage and both accumulators start empty
+    if (threadIdx.x == 0) {
         for (int st = 0; st < S; ++st) mbar_arrive(empty + st);
+        mbar_arrive(acc_empty + 0);
+        mbar_arrive(acc_empty + 1);
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
     const int pos0 = s_pos0;
     unsigned target = 0;
     int n_barrier = 0;
@@ -1147,8 +1188,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         if (n_barrier == 1 && blockIdx.x == 0 && threadIdx.x == 0) *p.seq = s_seq + 1u;
         return true;
     };
-    Pipe pp{full, empty, 0u, 0u};
+    Pipe pp{full, empty, acc_full, acc_empty, s_tmem, 0u, 0u, 0u, 0u, 0};
     bool prefetched = false;
+    bool failed = false;
     int attn_pre = 0;  // producer: K / V chunks of the next attention op requested early
     copy_op(p.ops, s_op);
     for (int o = 0; o < p.n_ops; ++o) {
@@ -1163,7 +1205,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         constexpr int kOpChunks = (int)(sizeof(FwdOp) / 16);
         static_assert(sizeof(FwdOp) % 16 == 0 && kOpChunks <= 32, "an op is copied in 16-byte pieces by one warp");
         const bool has_nx = o + 1 < p.n_ops;
-        const int plane = (int)threadIdx.x - kConsumers;  // lane in the producer warp
+        const int plane = mma_warp ? -1 : (int)threadIdx.x - kConsumers;  // lane in the producer warp
         if (has_nx && plane >= 0 && plane < kOpChunks)
             asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
                              smem_u32(reinterpret_cast<unsigned char*>(s_op + ((o + 1) & 1)) + 16 * plane)),
@@ -1194,12 +1236,12 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
             if (!ok) s_fail = 1;
             __syncthreads();
             if (s_fail) {
-                drain_before_exit();
-                return;
+                failed = true;
+                break;
             }
             if (!barrier_next()) {
-                drain_before_exit();
-                return;
+                failed = true;
+                break;
             }
             attn_combine<HD>(op.at, p.M, pos0);
         }
@@ -1224,18 +1266,29 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         if (!ok) s_fail = 1;
         __syncthreads();
         if (s_fail) {
-            drain_before_exit();
-            return;
+            failed = true;
+            break;
         }
         if (ct && threadIdx.x == 0) ct[4] = globaltimer();
         if (o + 1 < p.n_ops) {
             if (!barrier_next()) {
-                drain_before_exit();
-                return;
+                failed = true;
+                break;
             }
         }
         if (ct && threadIdx.x == 0) ct[5] = globaltimer();
         if (p.trace && blockIdx.x == 0 && threadIdx.x == 0) p.trace[o + 1] = globaltimer();
+    }
+    // After a failed wait, copies and MMAs still in flight get a bounded time
+    // to land; otherwise every MMA this CTA issued has completed (the
+    // consumers waited for each accumulator).  Then TMEM is freed.
+    if (failed) drain_before_exit();
+    tc_fence_before();
+    __syncthreads();
+    if (mma_warp) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(s_tmem), "r"(kTmemCols)
+                     : "memory");
     }
 }
 

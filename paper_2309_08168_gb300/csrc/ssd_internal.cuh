@@ -17,7 +17,9 @@ constexpr int kTileRows = 64;     // output rows per GEMM CTA
 constexpr int kGemmThreads = 256; // 8 warps: 4 row groups x 2 k-interleaves
 constexpr int kAttnChunk = 64;    // KV positions per attention CTA (absolute chunks)
 constexpr int kAttnThreads = 256;
-constexpr int kStreamKC = 256;    // k per streaming-GEMM work unit (64 rows x 256 = 32 KB of weights)
+constexpr int kStreamKC = 256;    // (stand-alone projection kernel of gemm.cu) k per CTA chunk step
+constexpr int kFTile = 128;       // forward kernel: weight rows per tile (tcgen05 M, TMEM lanes)
+constexpr int kFKC = 128;         // forward kernel: k per work unit (128 rows x 128 k = 32 KB of weights)
 constexpr int kTraceUnits = 1024, kTraceCtas = 1280;  // offsets in FwdParams::trace
 // rows per input plane of a forward of M rows (the plane classes)
 constexpr int fwd_plane_rows(int M) { return M == 1 ? 1 : (M <= 4 ? 4 : (M <= 8 ? 8 : (M <= 12 ? 12 : 16))); }

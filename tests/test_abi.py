@@ -50,8 +50,9 @@ def _cfg(ssd, **kw):
     return ssd.make_config(**base)
 
 
-@pytest.mark.parametrize("bad", [dict(head_dim=96), dict(n_kv_heads=3), dict(d_model=200), dict(ffn=100),
-                                 dict(vocab=40000), dict(max_seq=1), dict(n_layers=0)])
+@pytest.mark.parametrize("bad", [dict(head_dim=96), dict(n_kv_heads=3), dict(d_model=200), dict(d_model=320),
+                                 dict(ffn=100), dict(vocab=40000), dict(max_seq=1), dict(n_layers=0),
+                                 dict(n_heads=3, n_kv_heads=1)])
 def test_create_rejects_bad_config(ssd, bad):
     w = ssd.ssd_weights()  # all NULL: config is checked first, no device touched
     with pytest.raises(ssd.SSDError) as e:
