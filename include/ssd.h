@@ -213,13 +213,14 @@ int ssd_debug_time_forward(ssd_handle* h, int draft, int rows, int gemm_only, in
  * enough.  detail_op: index of one op to trace in detail (-1: none).
  * unit_trace (may be NULL): 256 globaltimer stamps (ns) of CTA 0 for
  * detail_op.  A projection: its first 64 work units, 4 per unit: producer
- * issue, consumer data ready, MMA done, segment flush done (0 if none).
+ * issue, MMAs issued, 0, segment flush done (0 if none).
  * Attention: its first 31 items, 8 per item: item start, q loaded, K / V
  * ready, after the CTA barrier, scores done, softmax done, P V done, 0; then
  * [248] partials published, [249] head counts added, [250] combine done.
  * cta_trace (may be NULL): 8 stamps per CTA of the forward kernel for
- * detail_op: op start, first data ready, last MMA done, work done, grid
- * barrier arrive, barrier release, number of work units, 0; max_ctas >= the
+ * detail_op: op start, first data ready (attention), last accumulator ready
+ * (projections) or last item done (attention), work done, grid barrier
+ * arrive, barrier release, number of work units (items), 0; max_ctas >= the
  * grid (the SM count), *n_ctas = the grid.
  * Errors: INVALID_ARG, CUDA. */
 int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, int* op_types,

@@ -607,7 +607,7 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 
         // RESID: this tile's residual h (written by earlier ops: L2), loaded
         // before waiting for the other segments so its latency overlaps it
-        constexpr int HJ = kMaxRows * kFTile / kGemmThreads;
+        constexpr int HJ = (R * kFTile + kGemmThreads - 1) / kGemmThreads;  // elements per thread (M <= R)
         float hpre[HJ], gpre[HJ];
         if (epi == EPI_RESID) {
 #pragma unroll
@@ -621,26 +621,44 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         }
 
         if (nseg > 1) {
-            // the other segments come from later CTAs, which never wait on this one
-            for (int idx = threadIdx.x; idx < M * kFTile; idx += kGemmThreads) {
+            // the other segments come from later CTAs, which never wait on this
+            // one.  Each thread issues the words of all its elements for a batch
+            // of segments before using any (one L2 round trip per batch), then
+            // adds them in segment order.
+            float acc[HJ];
+            int at[HJ];
+#pragma unroll
+            for (int j = 0; j < HJ; ++j) {
+                const int idx = threadIdx.x + j * kGemmThreads;
                 const int m = idx / kFTile, r = idx - m * kFTile;
-                const unsigned long long* p = slots + m * kFTile + r;
-                float sum = ys[r * 16 + m];
-                for (int sg0 = 1; sg0 < nseg; sg0 += 4) {
-                    unsigned long long w[4];
-#pragma unroll
-                    for (int j = 0; j < 4; ++j)
-                        if (sg0 + j < nseg) w[j] = ld_relaxed_u64(p + (size_t)(sg0 + j) * kSlot);
-#pragma unroll
-                    for (int j = 0; j < 4; ++j)
-                        if (sg0 + j < nseg) {
-                            if (tag_of(w[j]) != tag && !wait_tag(p + (size_t)(sg0 + j) * kSlot, tag, w[j], err))
-                                ok = false;
-                            sum += value_of(w[j]);
-                        }
-                }
-                ys[r * 16 + m] = sum;
+                at[j] = idx < M * kFTile ? m * kFTile + r : -1;
+                acc[j] = at[j] >= 0 ? ys[r * 16 + m] : 0.f;
             }
+            constexpr int QB = R <= 8 ? 4 : 2;  // segments per batch (registers: QB * HJ words)
+            for (int sg0 = 1; sg0 < nseg; sg0 += QB) {
+                unsigned long long w[QB][HJ];
+#pragma unroll
+                for (int q = 0; q < QB; ++q)
+#pragma unroll
+                    for (int j = 0; j < HJ; ++j)
+                        if (sg0 + q < nseg && at[j] >= 0) w[q][j] = ld_relaxed_u64(slots + (size_t)(sg0 + q) * kSlot + at[j]);
+#pragma unroll
+                for (int q = 0; q < QB; ++q)
+#pragma unroll
+                    for (int j = 0; j < HJ; ++j)
+                        if (sg0 + q < nseg && at[j] >= 0) {
+                            unsigned long long wv = w[q][j];
+                            if (tag_of(wv) != tag && !wait_tag(slots + (size_t)(sg0 + q) * kSlot + at[j], tag, wv, err))
+                                ok = false;
+                            acc[j] += value_of(wv);
+                        }
+            }
+#pragma unroll
+            for (int j = 0; j < HJ; ++j)
+                if (at[j] >= 0) {
+                    const int m = at[j] / kFTile, r = at[j] - m * kFTile;
+                    ys[r * 16 + m] = acc[j];
+                }
             consumer_sync();
         }
 
@@ -841,7 +859,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
     constexpr int QST = L::QST, PST = L::PST;
     __half* qh = reinterpret_cast<__half*>(smem + L::ATT);  // [VG][QST] q hi, then lo
     __half* ql = qh + VG * QST;
-    float* sc = reinterpret_cast<float*>(smem + L::ATT_SC);  // [VG][SP] scores
+    float* sc = reinterpret_cast<float*>(smem + L::ATT_SC);  // per-warp maxima and sums
     __half* ph = reinterpret_cast<__half*>(smem + L::ATT_P);  // [VG][PST] weights hi, then lo
     __half* pl = ph + VG * PST;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -907,7 +925,13 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
         stamp(it, 3);
 
         // scores S = K q^T on tensor cores: warp w takes positions 16w..16w+15
-        // (A = K rows, 128-byte swizzled), all 16 vectors (B = q hi, then lo)
+        // (A = K rows, 128-byte swizzled), all 16 vectors (B = q hi, then lo);
+        // then the softmax of every vector over the segment straight from the
+        // accumulators: per-warp maxima -> CTA barrier -> the segment maximum
+        // (the 8 warps' values in order) -> weights as fp16 hi + lo, per-warp
+        // sums (the partial's sum adds the 8 warps' sums in order)
+        float* wmax = sc;           // [8 warps][VG vectors]
+        float* wsum = sc + 8 * VG;  // [8 warps][VG vectors]
         {
             const int p0 = warp * 16, j = p0 / kAttnChunk;
             float c[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
@@ -938,39 +962,60 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
                     const int vl = nt * 8 + 2 * tg + (x & 1), pq = p0 + g + 8 * (x >> 1);
                     const int m = (v0 + vl) / G;
                     const bool vis = j < n_u && vl < nv && t0 + pq <= pos0 + m;
-                    sc[vl * SP + pq] = vis ? c[nt][x] * a.scale : -INFINITY;
+                    c[nt][x] = vis ? c[nt][x] * a.scale : -INFINITY;
+                }
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int cx = 0; cx < 2; ++cx) {
+                    float v = fmaxf(c[nt][cx], c[nt][cx + 2]);
+                    v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
+                    v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
+                    v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 16));
+                    if (g == 0) wmax[warp * VG + nt * 8 + 2 * tg + cx] = v;
+                }
+            consumer_sync();
+            stamp(it, 4);
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int cx = 0; cx < 2; ++cx) {
+                    const int vl = nt * 8 + 2 * tg + cx;
+                    float mx = -INFINITY;
+#pragma unroll
+                    for (int w2 = 0; w2 < kConsumers / 32; ++w2) mx = fmaxf(mx, wmax[w2 * VG + vl]);
+                    float l = 0.f;
+#pragma unroll
+                    for (int xh = 0; xh < 2; ++xh) {
+                        const float x = c[nt][cx + 2 * xh];
+                        const float pq = x == -INFINITY ? 0.f : expf(x - mx);
+                        const __half hh = __float2half_rn(pq);
+                        const int pos = p0 + g + 8 * xh;
+                        ph[vl * PST + pos] = hh;
+                        pl[vl * PST + pos] = __float2half_rn(pq - __half2float(hh));
+                        l += pq;
+                    }
+                    l += __shfl_xor_sync(0xffffffffu, l, 4);
+                    l += __shfl_xor_sync(0xffffffffu, l, 8);
+                    l += __shfl_xor_sync(0xffffffffu, l, 16);
+                    if (g == 0) wsum[warp * VG + vl] = l;
                 }
         }
         consumer_sync();
-        stamp(it, 4);
-
-        // softmax over the segment: warp per vector; weights as fp16 hi + lo
-        for (int vl = warp; vl < nv; vl += kConsumers / 32) {
-            const int v = v0 + vl, m = v / G;
-            float* o = part + (size_t)v * part_v;
-            const float* sv = sc + vl * SP;
-            float mx = -INFINITY;
-#pragma unroll
-            for (int q = 0; q < SP / 32; ++q) mx = fmaxf(mx, sv[lane + 32 * q]);
-            mx = warp_max(mx);
-            float l = 0.f;
-#pragma unroll
-            for (int q = 0; q < SP / 32; ++q) {
-                const float x = sv[lane + 32 * q];
-                const float pq = x == -INFINITY ? 0.f : expf(x - mx);
-                const __half hh = __float2half_rn(pq);
-                ph[vl * PST + lane + 32 * q] = hh;
-                pl[vl * PST + lane + 32 * q] = __float2half_rn(pq - __half2float(hh));
-                l += pq;
-            }
-            l = warp_sum(l);
-            if (lane == 0) {
-                o[HD] = pos0 + m < t0 ? -INFINITY : mx;  // -inf: nothing visible in this segment
-                o[HD + 1] = l;
-            }
-        }
-        consumer_sync();
         stamp(it, 5);
+        // the segment's (max, sum) of each vector; -inf: nothing visible
+        if (tid < nv) {
+            const int v = v0 + tid, m = v / G;
+            float mx = -INFINITY, l = 0.f;
+#pragma unroll
+            for (int w2 = 0; w2 < kConsumers / 32; ++w2) {
+                mx = fmaxf(mx, wmax[w2 * VG + tid]);
+                l += wsum[w2 * VG + tid];
+            }
+            float* o = part + (size_t)v * part_v;
+            o[HD] = pos0 + m < t0 ? -INFINITY : mx;
+            o[HD + 1] = l;
+        }
 
         // O = P V on tensor cores: warp w takes dims 16w..16w+15 (B = V rows via
         // transposed 8x8 loads), all 16 vectors (A = P hi, then lo); rows of
@@ -1017,22 +1062,25 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
 // Second phase of attention, after a grid barrier (the segment partials of
 // every CTA are visible): the partials of each (KV head, query vector) are
 // combined in segment order - row m uses segments 0 .. (pos0 + m) / SP - and
-// written as the bf16 hi / lo planes of the attention output.  The outputs
-// are spread over every CTA's consumer threads, one thread per 4 dims of a
-// vector (consecutive threads: consecutive dims, coalesced loads), so the
-// combine costs about two dependent L2 round trips whatever the number of
-// vectors and segments.
+// written as the bf16 hi / lo planes of the attention output.  One warp (half
+// a warp at head_dim 64) per vector, 4 dims per thread (coalesced loads), the
+// vectors spread round-robin over the warps of all CTAs, so the combine
+// costs about two dependent L2 round trips whatever the number of vectors
+// and segments, and no SM carries much of its traffic.
 template <int HD>
 __device__ void attn_combine(const AttnArgs& a, int M, int pos0) {
     if (threadIdx.x >= kConsumers) return;
-    constexpr int SP = kAttnSegChunks * kAttnChunk, HD4 = HD / 4;
+    constexpr int SP = kAttnSegChunks * kAttnChunk, HD4 = HD / 4, VPW = 32 / HD4;  // vectors per warp
     const int G = a.n_heads / a.n_kv_heads, NV = G * M;
-    const size_t part_v = HD + 2;              // floats per partial: o[HD], max, sum
+    const size_t part_v = HD + 2;                  // floats per partial: o[HD], max, sum
     const size_t qs_stride = (size_t)NV * part_v;  // next segment of the same vector
-    const int tasks = a.n_kv_heads * NV * HD4;
-    for (int k = blockIdx.x * kConsumers + threadIdx.x; k < tasks; k += gridDim.x * kConsumers) {
-        const int kvh = k / (NV * HD4), r = k - kvh * NV * HD4;
-        const int v = r / HD4, e = (r - v * HD4) * 4;
+    const int n_vec = a.n_kv_heads * NV;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int n_warps = gridDim.x * (kConsumers / 32);
+    // warp-major over the CTAs: the first vectors go to warp 0 of every CTA
+    for (int gv = (warp * gridDim.x + blockIdx.x) * VPW + lane / HD4; gv < n_vec; gv += n_warps * VPW) {
+        const int kvh = gv / NV, v = gv - kvh * NV;
+        const int e = (lane % HD4) * 4;
         const int m = v / G, gi = v - m * G;
         const int nsg = (pos0 + m) / SP + 1;
         const float* pv = a.part + (size_t)kvh * a.n_chunks * qs_stride + (size_t)v * part_v;
