@@ -119,24 +119,6 @@ __device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long
     asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
     return v;
 }
-// Bounded wait until the word at p carries `tag` (w: the word read); false
-// (timeout recorded) after kBarrierTimeoutNs or when another CTA already
-// recorded an error.  Kept out of line: inlined into the projection op, this
-// cold loop measurably slowed its MMA loop.
-__device__ __noinline__ bool wait_tag(const unsigned long long* p, unsigned tag, unsigned long long& w, int* err) {
-    const unsigned long long t0 = globaltimer();
-    for (;;) {
-        __nanosleep(32);
-        w = ld_relaxed_u64(p);
-        if (tag_of(w) == tag) return true;
-        if (*(volatile int*)err) return false;
-        if (globaltimer() - t0 > kBarrierTimeoutNs) {
-            atomicCAS(err, 0, kDevErrTimeout);
-            return false;
-        }
-    }
-}
-
 __device__ __forceinline__ int unit_owner(long long u, long long U, long long G) {
     return (int)(((u + 1) * G + U - 1) / U - 1);
 }
@@ -642,16 +624,38 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 #pragma unroll
                     for (int j = 0; j < HJ; ++j)
                         if (sg0 + q < nseg && at[j] >= 0) w[q][j] = ld_relaxed_u64(slots + (size_t)(sg0 + q) * kSlot + at[j]);
+                // words that do not carry this op's tag yet (their segment's CTA
+                // has not published) are re-read together, not one at a time
+                unsigned long long t_wait = 0;
+                for (;;) {
+                    bool ready = true;
+#pragma unroll
+                    for (int q = 0; q < QB; ++q)
+#pragma unroll
+                        for (int j = 0; j < HJ; ++j)
+                            if (sg0 + q < nseg && at[j] >= 0 && tag_of(w[q][j]) != tag) ready = false;
+                    if (ready) break;
+                    const unsigned long long now = globaltimer();
+                    if (t_wait == 0) t_wait = now;
+                    if (*(volatile int*)err) { ok = false; break; }
+                    if (now - t_wait > kBarrierTimeoutNs) {
+                        atomicCAS(err, 0, kDevErrTimeout);
+                        ok = false;
+                        break;
+                    }
+                    __nanosleep(64);
+#pragma unroll
+                    for (int q = 0; q < QB; ++q)
+#pragma unroll
+                        for (int j = 0; j < HJ; ++j)
+                            if (sg0 + q < nseg && at[j] >= 0 && tag_of(w[q][j]) != tag)
+                                w[q][j] = ld_relaxed_u64(slots + (size_t)(sg0 + q) * kSlot + at[j]);
+                }
 #pragma unroll
                 for (int q = 0; q < QB; ++q)
 #pragma unroll
                     for (int j = 0; j < HJ; ++j)
-                        if (sg0 + q < nseg && at[j] >= 0) {
-                            unsigned long long wv = w[q][j];
-                            if (tag_of(wv) != tag && !wait_tag(slots + (size_t)(sg0 + q) * kSlot + at[j], tag, wv, err))
-                                ok = false;
-                            acc[j] += value_of(wv);
-                        }
+                        if (sg0 + q < nseg && at[j] >= 0) acc[j] += value_of(w[q][j]);
             }
 #pragma unroll
             for (int j = 0; j < HJ; ++j)
