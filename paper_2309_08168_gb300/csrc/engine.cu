@@ -96,7 +96,7 @@ struct ssd_handle {
     float* h = nullptr;
     bf16* xn_hi = nullptr;  // planes of h * g (input of the next normed projection) [2][16][d]
     bf16* xn_lo = nullptr;  // = xn_hi + 16 * d
-    float* ss = nullptr;    // per-64-column sums of h^2 [16][d/64]
+    float* ss = nullptr;    // per-128-column sums of h^2 [16][d/128]
     float* q = nullptr;
     bf16* at_hi = nullptr;  // attention output planes [16][H*hd]
     bf16* at_lo = nullptr;
@@ -348,7 +348,7 @@ GemmArgs proj_args(ssd_handle* h, int N, int K, int n_tiles, const bf16* x_hi, c
 // The op list of one forward: embedding, the sublayers that run (all of them,
 // or those outside the skip set for the draft model), lm_head last.
 // RMSNorm is folded into the projections: whoever produces the residual
-// stream also writes the bf16 hi / lo planes of h * g_next and per-64-column
+// stream also writes the bf16 hi / lo planes of h * g_next and per-128-column
 // sums of h^2; the consuming projection scales row m by rsqrt(mean(h^2) + eps).
 std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
     const ssd_config& c = h->cfg;

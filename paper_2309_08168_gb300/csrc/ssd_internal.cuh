@@ -13,7 +13,7 @@ typedef __half f16;
 
 constexpr int kMaxRows = 16;      // rows of one forward (verification K+1 <= 16)
 constexpr int kMaxK = 15;         // drafts per round
-constexpr int kTileRows = 64;     // output rows per GEMM CTA
+constexpr int kTileRows = 64;     // stand-alone projection kernel (gemm.cu): output rows per CTA
 constexpr int kGemmThreads = 256; // 8 warps: 4 row groups x 2 k-interleaves
 constexpr int kAttnChunk = 64;    // KV positions per attention CTA (absolute chunks)
 constexpr int kAttnThreads = 256;
@@ -51,7 +51,8 @@ struct DecodeState {
 };
 
 // ---------------------------------------------------------------------------
-// GEMM (swap-AB skinny GEMM on mma.sync m16n8k16, bf16 in, fp32 accumulate)
+// Projection arguments: the forward kernel's tcgen05 projections and the
+// stand-alone swap-AB mma.sync kernel of gemm.cu (bf16 in, fp32 accumulate)
 // ---------------------------------------------------------------------------
 enum GemmEpi { EPI_LOGITS = 0, EPI_RESID = 1, EPI_SWIGLU = 2, EPI_QKV = 3 };
 
@@ -67,7 +68,7 @@ struct GemmArgs {
     const float* x;      // activations [M][K] fp32 (split into bf16 hi + lo in the kernel)
     int M;               // activation rows (1..16)
     float* partial;      // split-K partials: gemm.cu [ksplit][M][n_tiles*64] floats; forward
-                         // kernel [n_tiles][n_chunks][16][64] tagged 64-bit words
+                         // kernel [n_tiles][n_chunks][16][128] tagged 64-bit words
     unsigned* counters;  // gemm.cu: [n_tiles] arrival counters (left at zero); unused by the forward kernel
     // epilogue operands
     float* out_f32;      // EPI_LOGITS: [M][ldo]; EPI_RESID: residual h [M][ldo]
@@ -92,15 +93,13 @@ struct GemmArgs {
     bf16* xo_hi;         // EPI_RESID: planes of h * g_next [M][N]; EPI_SWIGLU: act planes [M][ffn]
     bf16* xo_lo;
     float* ss_out;       // EPI_RESID: [M][n_tiles] per-tile sums of h^2
-    int n_chunks;        // ceil(K / kStreamKC)
+    int n_chunks;        // forward kernel: ceil(K / kFKC)
     int n_units;         // n_tiles * n_chunks
-    // TMA tensor maps (in global memory).  wide = 1 (K % 64 == 0): w maps view
-    // W as {64, K/64, rows} with box {64, 4, 32} (one copy per 32-row half of
-    // a unit), x maps view the planes as {64, K/64, 16, 2} with box
-    // {64, 4, R, 2} (one copy per unit).  wide = 0: 2D w maps with box
-    // {64, 32} and 3D x maps {64, 16, 2} with box {64, R, 2}, one copy per
-    // 64-wide k-box.
-    int wide;
+    // TMA tensor maps (in global memory), forward kernel: w maps view W as
+    // {K, rows} with box {64, 128} (SwiGLU gate / up: {64, 64}), one copy per
+    // 64-wide k box of a unit; x maps view the planes as {K, 16, 2} with box
+    // {64, R, 2}, one copy per k box.
+    int wide;            // (unused by the forward kernel)
     const void* tm_w[3];  // w0, w1, w2
     const void* tm_x[kPlaneClasses];  // input planes for R = 1 | 4 | 8 | 12 | 16
 };
@@ -152,7 +151,7 @@ struct FwdParams {
     float* h;             // residual stream [16][d]
     bf16* xn_hi;          // planes of h * g [16][d]
     bf16* xn_lo;
-    float* ss;            // per-64-column sums of h^2 [16][d/64]
+    float* ss;            // per-128-column sums of h^2 [16][d/128]
     unsigned* bar;        // grid-barrier counter, zero at launch
     unsigned* seq;        // forward sequence number (tags split-K partials; +1 per launch)
     int* err;             // device error code
