@@ -269,7 +269,7 @@ struct GemmSmem {
     static constexpr int WB = kFTile * kFKC * 2;    // 32 KB of weights per unit
     static constexpr int XKB = NP * 128;            // input bytes per 64-wide k box
     static constexpr int STAGE = WB + 2 * XKB;
-    static constexpr int S = R <= 8 ? 5 : 4;        // ring depth
+    static constexpr int S = 5;                     // ring depth (160 KB of weights in flight)
     static constexpr int VG = 16;  // attention: query vectors per item (one MMA M / N tile)
     static constexpr int YS = S * STAGE;            // [128][16] floats: the finished segment
     // attention scratch: q hi / lo (fp16, rows padded by 16 bytes), scores
@@ -277,12 +277,13 @@ struct GemmSmem {
     static constexpr int QST = 128 + 8, PST = kAttnSegChunks * kAttnChunk + 8;  // halves per row
     static constexpr int ATT = S * STAGE;
     static constexpr int ATT_SC = ATT + 2 * VG * QST * 2;
-    static constexpr int ATT_P = ATT_SC + VG * kAttnSegChunks * kAttnChunk * 4;
+    static constexpr int ATT_P = ATT_SC + 2 * (kConsumers / 32) * VG * 4;  // per-warp maxima and sums
     static constexpr int SCRATCH_GEMM = kFTile * 16 * 4;
     static constexpr int SCRATCH_ATT = ATT_P + 2 * VG * PST * 2 - ATT;
     static constexpr size_t BYTES =
         1024 + (size_t)S * STAGE + (SCRATCH_GEMM > SCRATCH_ATT ? SCRATCH_GEMM : SCRATCH_ATT);
     static_assert(STAGE >= 2 * kAttnChunk * 128 * 2, "a stage holds the K and V rows of one 64-position chunk");
+    static_assert(BYTES + 4096 <= 232448, "dynamic + static shared memory within the per-CTA limit");
 };
 
 // ---------------------------------------------------------------------------
