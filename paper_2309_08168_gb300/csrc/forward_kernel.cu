@@ -83,9 +83,8 @@ __device__ bool grid_barrier(unsigned* bar, unsigned target, int* err, unsigned 
     __syncthreads();
     if (threadIdx.x == 0) {
         // the CTA's stores (ordered before this thread by the CTA barrier) are
-        // published by the fence; the arrival itself needs no reply
-        __threadfence();
-        asm volatile("red.relaxed.gpu.global.add.u32 [%0], 1;" ::"l"(bar) : "memory");
+        // published by the release of the arrival, which needs no reply
+        asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(bar) : "memory");
         int ok = 1;
         const unsigned long long t0 = globaltimer();
         while (ld_acquire(bar) < target) {  // acquire: later loads see the others' stores
