@@ -1367,16 +1367,6 @@ int configure_fwd() {
 
 }  // namespace
 
-size_t forward_smem_bytes(int M) {
-    switch (fwd_plane_rows(M)) {
-        case 1: return GemmSmem<1>::BYTES;
-        case 4: return GemmSmem<4>::BYTES;
-        case 8: return GemmSmem<8>::BYTES;
-        case 12: return GemmSmem<12>::BYTES;
-        default: return GemmSmem<16>::BYTES;
-    }
-}
-
 int forward_configure() {
     int e = 0;
     e = e ? e : configure_fwd<1, 64>();

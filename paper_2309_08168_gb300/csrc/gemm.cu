@@ -1,20 +1,12 @@
-// gemm.cu - skinny projection GEMM of the decode forward (draft, verification
-// and prefill), Y[M x N] = X[M x K] * W^T with W bf16 [N][K], M <= 16.
+// gemm.cu - the stand-alone skinny projection GEMM of ssd_linear_noalloc:
+// Y[M x N] = X[M x K] * W^T with W bf16 [N][K], fp32 X and Y, M <= 16.
 //
-// Every projection of the LLaMA-2 decoder (Sec. 4.1) runs through this one
-// kernel: the fused q/k/v projection with RoPE and the KV-cache write, the
-// output and down projections with the residual add, the gate/up projection
-// with SwiGLU, and the lm_head.  The weights are the large operand, so the
-// kernel is "swap-AB": 16 weight rows form the M side of an m16n8k16
-// tensor-core MMA and the <= 16 activation rows form its N side.
-//
-// Batch invariance (needed for greedy self-speculative output to be bit
-// identical to plain autoregressive output, Sec. 1 / App. G.2): the result
-// for activation row m depends only on row m.  The MMA computes every output
-// column independently, the split of K into CTA chunks, into k-interleaved
-// warps and into the fixed-order split-K combine depends on (N, K) only, and
-// every epilogue is element-wise per row.  So a verification row equals the
-// M = 1 forward of the same token at the same position bit for bit.
+// The weights are the large operand, so the kernel is "swap-AB": 16 weight
+// rows form the M side of an m16n8k16 tensor-core MMA and the <= 16
+// activation rows form its N side.  The result for activation row m depends
+// only on row m (the MMA computes every output column independently, and the
+// split of K into CTA chunks, into k-interleaved warps and into the
+// fixed-order split-K combine depends on (N, K) only).
 //
 // Precision: the fp32 activation rows are split into bf16 hi = rn(x) and
 // lo = rn(x - hi) and both are multiplied (the MMA's N side holds the hi rows
@@ -24,10 +16,9 @@
 // CTA = 256 threads: warp w handles the 16-row group (w & 3) of the 64-row
 // tile and the k32 blocks b = (w >> 2) (mod 2) of its k-chunk.  The weight
 // chunk (64 rows x kc) is streamed HBM -> shared memory with 16-byte cp.async,
-// then fed to
-// the MMA with a k-permutation: thread (g, t) reads 8 consecutive bf16 of a
-// row, which the A and B fragments both interpret as the same logical k
-// slots, so the product is unchanged and every load is a 128-bit LDS.
+// then fed to the MMA with a k-permutation: thread (g, t) reads 8 consecutive
+// bf16 of a row, which the A and B fragments both interpret as the same
+// logical k slots, so the product is unchanged and every load is a 128-bit LDS.
 #include <mutex>
 #include <string>
 
@@ -39,7 +30,7 @@ namespace {
 
 // NPH = n8 tiles per activation half (1: M <= 8, 2: M <= 16).  The MMA's N
 // side holds P = 8*NPH rows of x_hi followed by P rows of x_lo.
-template <int NPH, int EPI>
+template <int NPH>
 __global__ void __launch_bounds__(kGemmThreads) gemm_kernel(const GemmArgs a) {
     constexpr int NT = 2 * NPH;
     constexpr int P = 8 * NPH;
@@ -60,7 +51,8 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_kernel(const GemmArgs a) {
     const int cpr = kc_eff >> 3;  // 16-byte chunks per row
     for (int c = threadIdx.x; c < kTileRows * cpr; c += kGemmThreads) {
         int r = c / cpr, cc = c - r * cpr;
-        const bf16* src = row_src(a, EPI, tile, r);
+        const int n = tile * kTileRows + r;
+        const bf16* src = n < a.N ? a.w0 + (size_t)n * a.K : nullptr;
         const bf16* g = src ? src + k0 + cc * 8 : a.w0;
         SSD_GUARD(a.err, (((uintptr_t)g & 15u) == 0) && (r * pitch + cc * 16 + 16 <= kTileRows * pitch), 101)
         cp_async16(ws + r * pitch + cc * 16, g, src ? 16 : 0);
@@ -172,63 +164,15 @@ __global__ void __launch_bounds__(kGemmThreads) gemm_kernel(const GemmArgs a) {
         __syncthreads();
     }
 
-    // 6. epilogues (element-wise per activation row)
-    if (EPI == EPI_LOGITS || EPI == EPI_RESID) {
-        for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
-            int m = idx / kTileRows, r = idx - m * kTileRows;
-            int n = tile * kTileRows + r;
-            if (n >= a.N) continue;
-            float y = ys[r * 16 + m];
-            float* o = a.out_f32 + (size_t)m * a.ldo + n;
-            if (EPI == EPI_LOGITS) *o = y;
-            else *o = *o + y;
-        }
-    } else if (EPI == EPI_SWIGLU) {
-        for (int idx = threadIdx.x; idx < M * 32; idx += kGemmThreads) {
-            int m = idx >> 5, r = idx & 31;
-            int i = tile * 32 + r;
-            if (i >= a.ffn) continue;
-            float gt = ys[r * 16 + m], up = ys[(r + 32) * 16 + m];
-            a.out_act[(size_t)m * a.ffn + i] = gt / (1.f + expf(-gt)) * up;
-        }
-    } else {  // EPI_QKV
-        const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
-        const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
-        const int pos0 = a.st->pos0;
-        if (tile < q_tiles + k_tiles) {
-            const bool is_q = tile < q_tiles;
-            const int tt = is_q ? tile : tile - q_tiles;
-            const int head = tt / per_head, j0 = (tt % per_head) * 32;
-            for (int idx = threadIdx.x; idx < M * 32; idx += kGemmThreads) {
-                int m = idx >> 5, r = idx & 31;
-                int i = j0 + r, pos = pos0 + m;
-                float x1 = ys[r * 16 + m], x2 = ys[(r + 32) * 16 + m];
-                float2 cs = a.rope[(size_t)pos * half + i];
-                float y1 = x1 * cs.x - x2 * cs.y;
-                float y2 = x2 * cs.x + x1 * cs.y;
-                if (is_q) {
-                    float* q = a.q_out + (size_t)m * a.n_heads * hd + head * hd;
-                    q[i] = y1;
-                    q[i + half] = y2;
-                } else {
-                    f16* k = a.k_cache + ((size_t)head * a.max_seq + pos) * hd;
-                    k[i] = __float2half_rn(y1);
-                    k[i + half] = __float2half_rn(y2);
-                }
-            }
-        } else {
-            const int vt = tile - q_tiles - k_tiles;
-            for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
-                int m = idx / kTileRows, r = idx - m * kTileRows;
-                int f = vt * kTileRows + r;
-                int head = f / hd, e = f - head * hd;
-                a.v_cache[((size_t)head * a.max_seq + pos0 + m) * hd + e] = __float2half_rn(ys[r * 16 + m]);
-            }
-        }
+    // 6. the output rows
+    for (int idx = threadIdx.x; idx < M * kTileRows; idx += kGemmThreads) {
+        int m = idx / kTileRows, r = idx - m * kTileRows;
+        int n = tile * kTileRows + r;
+        if (n < a.N) a.out_f32[(size_t)m * a.ldo + n] = ys[r * 16 + m];
     }
 }
 
-template <int NPH, int EPI>
+template <int NPH>
 int launch_one(const GemmArgs& a, cudaStream_t s) {
     const size_t smem = gemm_smem_bytes(a.kc, a.M);
     cudaLaunchConfig_t cfg = {};
@@ -241,44 +185,25 @@ int launch_one(const GemmArgs& a, cudaStream_t s) {
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return (int)cudaLaunchKernelEx(&cfg, gemm_kernel<NPH, EPI>, a);
+    return (int)cudaLaunchKernelEx(&cfg, gemm_kernel<NPH>, a);
 }
 
-template <int NPH, int EPI>
+template <int NPH>
 int configure_one() {
-    return (int)cudaFuncSetAttribute(gemm_kernel<NPH, EPI>,
+    return (int)cudaFuncSetAttribute(gemm_kernel<NPH>,
                                      cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
 }
 
 }  // namespace
 
 int gemm_configure() {
-    int e = 0;
-    e = e ? e : configure_one<1, EPI_LOGITS>();
-    e = e ? e : configure_one<2, EPI_LOGITS>();
-    e = e ? e : configure_one<1, EPI_RESID>();
-    e = e ? e : configure_one<2, EPI_RESID>();
-    e = e ? e : configure_one<1, EPI_SWIGLU>();
-    e = e ? e : configure_one<2, EPI_SWIGLU>();
-    e = e ? e : configure_one<1, EPI_QKV>();
-    e = e ? e : configure_one<2, EPI_QKV>();
-    return e;
+    int e = configure_one<1>();
+    return e ? e : configure_one<2>();
 }
 
 size_t gemm_smem_bytes(int kc, int M) {
     const int P = gemm_half_rows(M);
     return (size_t)(kTileRows + 2 * P) * (kc * 2 + 64) + (size_t)kTileRows * 2 * P * sizeof(float);
-}
-
-int launch_gemm(int epi, const GemmArgs& a, cudaStream_t s) {
-    const bool two = a.M > 8;
-    switch (epi) {
-        case EPI_LOGITS: return two ? launch_one<2, EPI_LOGITS>(a, s) : launch_one<1, EPI_LOGITS>(a, s);
-        case EPI_RESID: return two ? launch_one<2, EPI_RESID>(a, s) : launch_one<1, EPI_RESID>(a, s);
-        case EPI_SWIGLU: return two ? launch_one<2, EPI_SWIGLU>(a, s) : launch_one<1, EPI_SWIGLU>(a, s);
-        case EPI_QKV: return two ? launch_one<2, EPI_QKV>(a, s) : launch_one<1, EPI_QKV>(a, s);
-    }
-    return (int)cudaErrorInvalidValue;
 }
 
 }  // namespace ssd
@@ -326,8 +251,8 @@ int noalloc_setup(int dev, NoAllocDevice** out) {
         cudaError_t e = cudaGetSymbolAddress((void**)&d.partial, g_noalloc_partial);
         if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&d.counters, g_noalloc_counters);
         if (e == cudaSuccess) e = cudaGetSymbolAddress((void**)&d.err, g_noalloc_err);
-        if (e == cudaSuccess) e = (cudaError_t)configure_one<1, EPI_LOGITS>();
-        if (e == cudaSuccess) e = (cudaError_t)configure_one<2, EPI_LOGITS>();
+        if (e == cudaSuccess) e = (cudaError_t)configure_one<1>();
+        if (e == cudaSuccess) e = (cudaError_t)configure_one<2>();
         // (the arrays start at zero when the module loads; each call clears
         // the counters it uses on its own stream)
         if (e != cudaSuccess)
@@ -386,7 +311,7 @@ extern "C" int ssd_linear_noalloc(const void* w, const float* x, float* y, int N
     a.ldo = N;
     a.err = d->err;
     if (e == cudaSuccess)
-        e = (cudaError_t)(M > 8 ? launch_one<2, EPI_LOGITS>(a, s) : launch_one<1, EPI_LOGITS>(a, s));
+        e = (cudaError_t)(M > 8 ? launch_one<2>(a, s) : launch_one<1>(a, s));
     if (e != cudaSuccess)
         return set_last_error(SSD_ERR_CUDA, (std::string("ssd_linear_noalloc: ") + cudaGetErrorString(e)).c_str());
 #ifdef SSD_CHECKED

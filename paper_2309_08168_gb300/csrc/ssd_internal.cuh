@@ -203,7 +203,6 @@ int prefill_configure();
 int prefill_chunk(const PrefillPlan& P, const int* toks, int n, int pos0, cudaStream_t s);
 
 int forward_configure();
-size_t forward_smem_bytes(int M);
 int launch_forward(const FwdParams& p, int head_dim, int grid, cudaStream_t s);
 
 // sets the thread's ssd_last_error() message and returns code
@@ -211,7 +210,6 @@ int set_last_error(int code, const char* msg);
 
 // launchers (return cudaError_t)
 int gemm_configure();
-int launch_gemm(int epi, const GemmArgs& a, cudaStream_t s);
 size_t gemm_smem_bytes(int kc, int M);
 constexpr int gemm_half_rows(int M) { return M <= 8 ? 8 : 16; }  // padded rows of x_hi (and of x_lo)
 
@@ -288,34 +286,6 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint3
         "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};\n"
         : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-
-// ---------------------------------------------------------------------------
-// GEMM helpers shared by both GEMM kernels
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ const bf16* row_src(const GemmArgs& a, int epi, int tile, int r) {
-    const int K = a.K;
-    if (epi == EPI_LOGITS || epi == EPI_RESID) {
-        int n = tile * kTileRows + r;
-        return n < a.N ? a.w0 + (size_t)n * K : nullptr;
-    }
-    if (epi == EPI_SWIGLU) {
-        int i = tile * 32 + (r & 31);
-        if (i >= a.ffn) return nullptr;
-        return (r < 32 ? a.w0 : a.w1) + (size_t)i * K;
-    }
-    // EPI_QKV: q and k tiles hold 32 RoPE pairs (i, i + hd/2) of one head
-    const int hd = a.head_dim, half = hd >> 1, per_head = hd / kTileRows;
-    const int q_tiles = a.n_heads * per_head, k_tiles = a.n_kv_heads * per_head;
-    if (tile < q_tiles + k_tiles) {
-        bool is_q = tile < q_tiles;
-        int tt = is_q ? tile : tile - q_tiles;
-        int head = tt / per_head, j0 = (tt % per_head) * 32;
-        int f = head * hd + (r >> 5) * half + j0 + (r & 31);
-        return (is_q ? a.w0 : a.w1) + (size_t)f * K;
-    }
-    int f = (tile - q_tiles - k_tiles) * kTileRows + r;
-    return a.w2 + (size_t)f * K;
 }
 
 // Splits 8 fp32 activations into bf16 hi = rn(x) and lo = rn(x - hi), so that
