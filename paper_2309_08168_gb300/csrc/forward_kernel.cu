@@ -352,6 +352,23 @@ __device__ __forceinline__ void tmem_ld<32>(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+template <>
+__device__ __forceinline__ void tmem_ld<24>(uint32_t taddr, float (&v)[24]) {
+    uint32_t r[24];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]),
+                   "=r"(r[23])
+                 : "r"(taddr + 16u));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 24; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 // Weight rows of tile t: one 128-row box (matrix s0 from row r0), or for
 // SwiGLU two 64-row boxes (the gate and the up rows of features 64 t ..).
 // The q / k / v widths are whole tiles, so a q / k tile is 128 / head_dim
@@ -546,9 +563,147 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         if (threadIdx.x == 0 && ct && i == n_my - 1) ct[6] = (unsigned long long)n_my;
         if (!(i == n_my - 1 || chunk == a.n_chunks - 1)) continue;
 
-        // this CTA's segment of the tile is complete: its accumulator holds
-        // W x_hi in columns 0..R-1 and W x_lo in columns R..2R-1
+        // this CTA's segment of the tile is complete (or completing): its
+        // accumulator holds W x_hi in columns 0..R-1 and W x_lo in columns
+        // R..2R-1.  Split-K: the CTA holding the tile's first chunks (its
+        // segment ends last, at the end of that CTA's range) finalises; the
+        // others store their partial and move on.  Each value travels with the
+        // op's tag in one 64-bit word, so the finaliser needs no flag and no
+        // fence: it reads each word until the tag is this op's.
         const int ab = pp.ab;
+        const long long u_first = (long long)tile * a.n_chunks;
+        const int seg0 = unit_owner(u_first, U, G);
+        const int nseg = unit_owner(u_first + a.n_chunks - 1, U, G) - seg0 + 1;
+        constexpr size_t kSlot = (size_t)kMaxRows * kFTile;
+        unsigned long long* slots =
+            reinterpret_cast<unsigned long long*>(a.partial) + (size_t)tile * a.n_chunks * kSlot;
+        const bool contributor = nseg > 1 && b != seg0;
+
+        if (contributor || epi == EPI_RESID) {
+            // Direct path: every consumer warp reads its own TMEM rows - warp w
+            // holds tile row rr = 32 (w % 4) + lane for the input rows m = w / 4,
+            // w / 4 + 2, ... - so nothing goes through shared memory and no CTA
+            // barrier precedes the stores.  A residual finaliser first fetches
+            // the residual rows, the gains and the other segments' partials
+            // while its own accumulator completes; its sum is own + (p_1 + p_2
+            // + ...), the partials added in segment order.
+            constexpr int HM = (R + 1) / 2;
+            const int q4 = warp & 3, par = warp >> 2, rr = q4 * 32 + lane;
+            const int n = tile * kFTile + rr;
+            float hp[HM], ps[HM];
+            const float gp = (!contributor && n < a.N && a.g_next) ? __bfloat162float(a.g_next[n]) : 0.f;
+#pragma unroll
+            for (int k = 0; k < HM; ++k) {
+                const int m = par + 2 * k;
+                hp[k] = (!contributor && m < M && n < a.N) ? __ldcg(a.out_f32 + (size_t)m * a.ldo + n) : 0.f;
+                ps[k] = 0.f;
+            }
+            if (!contributor && nseg > 1) {
+                constexpr int QB = R <= 8 ? 4 : R <= 12 ? 2 : 1;  // segments per batch (registers: QB * HM words)
+                for (int sg0 = 1; sg0 < nseg; sg0 += QB) {
+                    unsigned long long w[QB][HM];
+#pragma unroll
+                    for (int q = 0; q < QB; ++q)
+#pragma unroll
+                        for (int k = 0; k < HM; ++k)
+                            if (sg0 + q < nseg && par + 2 * k < M)
+                                w[q][k] = ld_relaxed_u64(slots + (size_t)(sg0 + q) * kSlot + (par + 2 * k) * kFTile + rr);
+                    // words that do not carry this op's tag yet (their CTA has
+                    // not published) are re-read together, not one at a time
+                    unsigned long long t_wait = 0;
+                    for (;;) {
+                        bool ready = true;
+#pragma unroll
+                        for (int q = 0; q < QB; ++q)
+#pragma unroll
+                            for (int k = 0; k < HM; ++k)
+                                if (sg0 + q < nseg && par + 2 * k < M && tag_of(w[q][k]) != tag) ready = false;
+                        if (ready) break;
+                        const unsigned long long now = globaltimer();
+                        if (t_wait == 0) t_wait = now;
+                        if (*(volatile int*)err) { ok = false; break; }
+                        if (now - t_wait > kBarrierTimeoutNs) {
+                            atomicCAS(err, 0, kDevErrTimeout);
+                            ok = false;
+                            break;
+                        }
+                        __nanosleep(64);
+#pragma unroll
+                        for (int q = 0; q < QB; ++q)
+#pragma unroll
+                            for (int k = 0; k < HM; ++k)
+                                if (sg0 + q < nseg && par + 2 * k < M && tag_of(w[q][k]) != tag)
+                                    w[q][k] = ld_relaxed_u64(slots + (size_t)(sg0 + q) * kSlot + (par + 2 * k) * kFTile + rr);
+                    }
+#pragma unroll
+                    for (int q = 0; q < QB; ++q)
+#pragma unroll
+                        for (int k = 0; k < HM; ++k)
+                            if (sg0 + q < nseg && par + 2 * k < M) ps[k] += value_of(w[q][k]);
+                }
+            }
+            ok = mbar_wait(pp.acc_full + ab, (pp.afull >> ab) & 1u, err) && ok;
+            pp.afull ^= 1u << ab;
+            pp.ab ^= 1;
+            tc_fence_after();
+            if (threadIdx.x == 0 && ct) ct[2] = globaltimer();
+            constexpr int NC = R == 12 ? 24 : NP;  // the 2R accumulator columns, rounded up
+            float v[NC];
+            tmem_ld<NC>(pp.tmem + (uint32_t)(ab * (kTmemCols / 2)) + ((uint32_t)(q4 * 32) << 16), v);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(pp.acc_empty + ab);  // this warp is done with the accumulator
+            float own[HM];
+#pragma unroll
+            for (int k = 0; k < HM; ++k) {  // input row m = par + 2k: columns m (hi) and R + m (lo)
+                const float hi = par ? v[(2 * k + 1) < NC ? 2 * k + 1 : 0] : v[2 * k];
+                const float lo = par ? v[(R + 2 * k + 1) < NC ? R + 2 * k + 1 : 0] : v[(R + 2 * k) < NC ? R + 2 * k : 0];
+                own[k] = hi + lo;
+            }
+            if (contributor) {
+                unsigned long long* mine = slots + (size_t)(b - seg0) * kSlot;
+#pragma unroll
+                for (int k = 0; k < HM; ++k)
+                    if (par + 2 * k < M) st_relaxed_u64(mine + (par + 2 * k) * kFTile + rr, tagged(tag, own[k]));
+                continue;
+            }
+            // residual finaliser: h += sum, the next norm's input planes of
+            // h * g_next and the per-tile sums of h^2 (per quadrant of 32 rows,
+            // then the 4 quadrants in order)
+            float* ssq = ys;  // [16][4]
+#pragma unroll
+            for (int k = 0; k < HM; ++k) {
+                const int m = par + 2 * k;
+                if (m >= M) break;  // (uniform in the warp)
+                float hv = 0.f;
+                if (n < a.N) {
+                    hv = hp[k] + (own[k] + ps[k]);
+                    a.out_f32[(size_t)m * a.ldo + n] = hv;
+                    if (a.g_next) {
+                        const float z = hv * gp;
+                        const bf16 zh = __float2bfloat16_rn(z);
+                        a.xo_hi[(size_t)m * a.N + n] = zh;
+                        a.xo_lo[(size_t)m * a.N + n] = __float2bfloat16_rn(z - __bfloat162float(zh));
+                    }
+                }
+                if (a.g_next) {
+                    const float sq = warp_sum(hv * hv);
+                    if (lane == 0) ssq[m * 4 + q4] = sq;
+                }
+            }
+            if (a.g_next) {
+                consumer_sync();
+                if (threadIdx.x < M)
+                    a.ss_out[threadIdx.x * a.n_tiles + tile] = (ssq[threadIdx.x * 4 + 0] + ssq[threadIdx.x * 4 + 1]) +
+                                                              (ssq[threadIdx.x * 4 + 2] + ssq[threadIdx.x * 4 + 3]);
+            }
+            consumer_sync();  // ys is reused by the next segment
+            if (ut && i < 64 && threadIdx.x == 0) ut[i * 4 + 3] = globaltimer();
+            continue;
+        }
+
+        // finalisers of the other epilogues: TMEM -> ys (warps 0-3), then the
+        // other segments' partials and the epilogue over ys
         ok = mbar_wait(pp.acc_full + ab, (pp.afull >> ab) & 1u, err) && ok;
         pp.afull ^= 1u << ab;
         pp.ab ^= 1;
@@ -563,44 +718,9 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
         }
         tc_fence_before();
         consumer_sync();
-        if (threadIdx.x == 0) mbar_arrive(pp.acc_empty + ab);  // the accumulator may be refilled
+        if (lane == 0) mbar_arrive(pp.acc_empty + ab);  // the accumulator may be refilled
 
-        // split-K: the CTA holding the tile's first chunks (its segment ends
-        // last, at the end of that CTA's range) finalises; the others store
-        // their partial and move on.  Each value travels with the op's tag in
-        // one 64-bit word, so the finaliser needs no flag and no fence: it
-        // reads each word until the tag is this op's.  The sum is in segment
-        // order.
-        const long long u_first = (long long)tile * a.n_chunks;
-        const int seg0 = unit_owner(u_first, U, G);
-        const int nseg = unit_owner(u_first + a.n_chunks - 1, U, G) - seg0 + 1;
-        constexpr size_t kSlot = (size_t)kMaxRows * kFTile;
-        unsigned long long* slots =
-            reinterpret_cast<unsigned long long*>(a.partial) + (size_t)tile * a.n_chunks * kSlot;
-        if (nseg > 1 && b != seg0) {
-            unsigned long long* mine = slots + (size_t)(b - seg0) * kSlot;
-            for (int idx = threadIdx.x; idx < M * kFTile; idx += kGemmThreads) {
-                const int m = idx / kFTile, r = idx - m * kFTile;
-                st_relaxed_u64(mine + m * kFTile + r, tagged(tag, ys[r * 16 + m]));
-            }
-            consumer_sync();  // ys is free for the next segment
-            continue;
-        }
-
-        // RESID: this tile's residual h (written by earlier ops: L2), loaded
-        // before waiting for the other segments so its latency overlaps it
         constexpr int HJ = (R * kFTile + kGemmThreads - 1) / kGemmThreads;  // elements per thread (M <= R)
-        float hpre[HJ], gpre[HJ];
-        if (epi == EPI_RESID) {
-#pragma unroll
-            for (int j = 0; j < HJ; ++j) {
-                const int idx = threadIdx.x + j * kGemmThreads;
-                const int m = idx / kFTile, n = tile * kFTile + (idx - m * kFTile);
-                const bool in = idx < M * kFTile && n < a.N;
-                hpre[j] = in ? __ldcg(a.out_f32 + (size_t)m * a.ldo + n) : 0.f;
-                gpre[j] = (in && a.g_next) ? __bfloat162float(a.g_next[n]) : 0.f;
-            }
-        }
 
         if (nseg > 1) {
             // the other segments come from later CTAs, which never wait on this
@@ -672,35 +792,6 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
                 const int m = idx / kFTile, r = idx - m * kFTile;
                 const int n = tile * kFTile + r;
                 if (n < a.N) a.out_f32[(size_t)m * a.ldo + n] = ys[r * 16 + m] * r_s[m];
-            }
-        } else if (epi == EPI_RESID) {
-#pragma unroll
-            for (int j = 0; j < HJ; ++j) {
-                const int idx = threadIdx.x + j * kGemmThreads;
-                if (idx >= M * kFTile) break;
-                const int m = idx / kFTile, r = idx - m * kFTile;
-                const int n = tile * kFTile + r;
-                float hv = 0.f;
-                if (n < a.N) {
-                    float* o = a.out_f32 + (size_t)m * a.ldo + n;
-                    hv = hpre[j] + ys[r * 16 + m];
-                    *o = hv;
-                    if (a.g_next) {
-                        const float z = hv * gpre[j];
-                        const bf16 zh = __float2bfloat16_rn(z);
-                        a.xo_hi[(size_t)m * a.N + n] = zh;
-                        a.xo_lo[(size_t)m * a.N + n] = __float2bfloat16_rn(z - __bfloat162float(zh));
-                    }
-                }
-                ys[r * 16 + m] = hv * hv;
-            }
-            if (a.g_next) {
-                consumer_sync();
-                for (int m = warp; m < M; m += kGemmThreads / 32) {
-                    const float sq = warp_sum((ys[lane * 16 + m] + ys[(lane + 32) * 16 + m]) +
-                                              (ys[(lane + 64) * 16 + m] + ys[(lane + 96) * 16 + m]));
-                    if (lane == 0) a.ss_out[m * a.n_tiles + tile] = sq;
-                }
             }
         } else if (epi == EPI_SWIGLU) {
             for (int idx = threadIdx.x; idx < M * 64; idx += kGemmThreads) {
@@ -1202,7 +1293,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(acc_full + b, 1);
-            mbar_init(acc_empty + b, 1);
+            mbar_init(acc_empty + b, kConsumers / 32);  // one arrival per consumer warp
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -1217,8 +1308,9 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
     // every stage and both accumulators start empty
-    if (threadIdx.x == 0) {
+    if (threadIdx.x == 0)
         for (int st = 0; st < S; ++st) mbar_arrive(empty + st);
+    if (threadIdx.x < kConsumers && (threadIdx.x & 31) == 0) {
         mbar_arrive(acc_empty + 0);
         mbar_arrive(acc_empty + 1);
     }
