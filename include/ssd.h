@@ -210,18 +210,20 @@ int ssd_debug_time_forward(ssd_handle* h, int draft, int rows, int gemm_only, in
  * of op o-1 to the end of op o, grid barrier included), op_types[o] = 0
  * embedding, 1 q/k/v projection, 2 attention, 3 output or down projection,
  * 4 gate/up projection, 5 lm_head.  max_ops >= 2 + 5 * n_layers is always
- * enough.  detail_op: index of one op to trace in detail (-1: none).
- * unit_trace (may be NULL): 256 globaltimer stamps (ns) of CTA 0 for
- * detail_op.  A projection: its first 64 work units, 4 per unit: producer
+ * enough.  detail_op: -1 (none), or the index of one op to trace in detail
+ * plus 65536 x the CTA whose unit stamps are taken (0 for CTA 0).
+ * unit_trace (may be NULL): 256 globaltimer stamps (ns) of that CTA for
+ * that op.  A projection: its first 64 work units, 4 per unit: producer
  * issue, MMAs issued, 0, segment flush done (0 if none).
  * Attention: its first 31 items, 8 per item: item start, q loaded, K / V
- * ready, after the CTA barrier, scores done, softmax done, P V done, 0; then
- * [248] partials published, [249] head counts added, [250] combine done.
+ * ready, after the CTA barrier, scores done, softmax done, P V done, 0.
  * cta_trace (may be NULL): 8 stamps per CTA of the forward kernel for
- * detail_op: op start, first data ready (attention), last accumulator ready
- * (projections) or last item done (attention), work done, grid barrier
- * arrive, barrier release, number of work units (items), 0; max_ctas >= the
- * grid (the SM count), *n_ctas = the grid.
+ * detail_op: [0] op start, [1] first data ready (attention), [2] last
+ * accumulator ready (projections) or arrival at the grid barrier between the
+ * segment partials and their combine (attention), [3] work done, [4] grid
+ * barrier arrive, [5] barrier release, [6] number of work units (items),
+ * [7] release of the attention's inner grid barrier (0 for projections);
+ * max_ctas >= the grid (the SM count), *n_ctas = the grid.
  * Errors: INVALID_ARG, CUDA. */
 int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, int* op_types,
                             int max_ops, int* n_ops, int detail_op, unsigned long long* unit_trace,

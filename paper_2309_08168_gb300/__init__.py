@@ -201,11 +201,11 @@ OP_NAMES = ("embed", "qkv", "attention", "o/down", "gate/up", "lm_head")
 
 def ssd_debug_trace_forward(h: int, draft: bool, rows: int, detail_op: int = -1):
     """Returns [(op name, microseconds)] for one forward of the forward kernel.
-    With detail_op >= 0 it returns (ops, units, ctas): units = [64][4] stamps
-    (ns) of CTA 0's first work units of that op (producer issue, MMAs issued,
-    0, segment flush done), ctas = [grid][8] stamps per CTA (op start, first
-    data ready (attention), last accumulator ready, work done, barrier
-    arrive, barrier release, units, 0)."""
+    With detail_op >= 0 (op index + 65536 x a CTA index) it returns (ops,
+    units, ctas): units = [64][4] stamps (ns) of that CTA's first work units
+    of that op (producer issue, MMAs issued, 0, segment flush done; for
+    attention 8 stamps per item), ctas = [grid][8] stamps per CTA in the
+    order ssd.h lists."""
     cfg = config_of(h)
     cap = 2 + 5 * cfg.n_layers
     us = np.zeros(cap, dtype=np.float32)

@@ -1132,6 +1132,8 @@ int ssd_debug_trace_forward(ssd_handle* h, int draft, int rows, float* op_us, in
     if (max_ops < n_ops) return fail(SSD_ERR_INVALID_ARG, "max_ops smaller than the op list");
     CUDA_TRY(cudaSetDevice(h->device), "set device");
     if (cta_trace && (!n_ctas || max_ctas < h->n_sms)) return fail(SSD_ERR_INVALID_ARG, "max_ctas below the grid");
+    if (detail_op >= 0 && ((detail_op & 0xffff) >= n_ops || (detail_op >> 16) >= h->n_sms))
+        return fail(SSD_ERR_INVALID_ARG, "detail_op: op index below the op count, CTA below the grid");
     cudaGraphExec_t traced = nullptr;
     int n = 0;
     h->trace_op = detail_op;

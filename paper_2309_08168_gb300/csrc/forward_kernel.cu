@@ -74,32 +74,29 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
     return v;
 }
 
-// Grid-wide barrier for a cooperative launch (all CTAs co-resident).  The
+// Grid-wide barrier for a cooperative launch (all CTAs co-resident), in two
+// halves so that a CTA can do work that publishes nothing between them.  The
 // counter only grows during a launch; `target` = gridDim.x * (barrier index).
-// Returns false (and records SSD_DEV_ERR_TIMEOUT) if the others do not arrive
-// within limit_ns, or if another CTA already gave up.
-__device__ bool grid_barrier(unsigned* bar, unsigned target, int* err, unsigned long long limit_ns) {
-    __shared__ int s_ok;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        // the CTA's stores (ordered before this thread by the CTA barrier) are
-        // published by the release of the arrival, which needs no reply
-        asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(bar) : "memory");
-        int ok = 1;
-        const unsigned long long t0 = globaltimer();
-        while (ld_acquire(bar) < target) {  // acquire: later loads see the others' stores
-            if (*(volatile int*)err) { ok = 0; break; }
-            if (globaltimer() - t0 > limit_ns) {
-                atomicCAS(err, 0, kDevErrTimeout);
-                ok = 0;
-                break;
-            }
-            __nanosleep(32);
+// grid_arrive (one thread, after a CTA barrier that orders the CTA's stores
+// before it): the release of the arrival publishes those stores and needs no
+// reply.  grid_wait (the same thread): acquire - later loads, ordered after it
+// by a CTA barrier, see the others' stores.  Returns false (and records
+// SSD_DEV_ERR_TIMEOUT) if the others do not arrive within limit_ns, or if
+// another CTA already gave up.
+__device__ __forceinline__ void grid_arrive(unsigned* bar) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(bar) : "memory");
+}
+__device__ bool grid_wait(unsigned* bar, unsigned target, int* err, unsigned long long limit_ns) {
+    const unsigned long long t0 = globaltimer();
+    while (ld_acquire(bar) < target) {
+        if (*(volatile int*)err) return false;
+        if (globaltimer() - t0 > limit_ns) {
+            atomicCAS(err, 0, kDevErrTimeout);
+            return false;
         }
-        s_ok = ok;
+        __nanosleep(32);
     }
-    __syncthreads();
-    return s_ok != 0;
+    return true;
 }
 
 // Split-K partials: a float and the tag of the op that wrote it (forward
@@ -1147,10 +1144,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
             for (int j = 0; j < n_u; ++j) mbar_arrive(pp.empty + (i + j) % S);  // the stages are free
         i += n_u;
     }
-    if (ct && tid == 0 && ar.i_begin < ar.i_end) {
-        ct[2] = globaltimer();
-        ct[6] = (unsigned long long)(ar.i_end - ar.i_begin);
-    }
+    if (ct && tid == 0) ct[6] = (unsigned long long)(ar.i_end - ar.i_begin);
     return ok;
 }
 
@@ -1265,7 +1259,7 @@ template <int R, int HD>
 __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams p) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
     __shared__ float r_s[kMaxRows];
-    __shared__ int s_pos0, s_fail, s_skip;
+    __shared__ int s_pos0, s_skip;
     __shared__ unsigned s_seq;
     __shared__ uint32_t s_tmem;
     constexpr int S = GemmSmem<R>::S;
@@ -1283,7 +1277,6 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         else if (p.src == SRC_DRAFT) pos0 = p.st->len + p.st->j;
         else pos0 = p.st->len;
         s_pos0 = pos0;
-        s_fail = 0;
         // a draft step after the round's drafting stage ended (draft exit): no work
         s_skip = p.src == SRC_DRAFT && *(volatile int*)&p.st->exited;
         s_seq = *(volatile unsigned*)p.seq;  // this forward's number (advanced by CTA 0 below)
@@ -1320,17 +1313,24 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
     const int pos0 = s_pos0;
     unsigned target = 0;
     int n_barrier = 0;
-    // Next grid barrier of this launch.  The profiling hook p.stall_barrier
-    // (0: none) makes barrier number n unreachable, so that its bounded wait
-    // runs out and the launch ends with the timeout recorded.
-    auto barrier_next = [&]() -> bool {
+    // Grid barriers of this launch, each split in two: thread 0 arrives right
+    // after a CTA barrier that ends the work before it, and waits for the
+    // others later, so the producer's requests for the next op (the issue of
+    // which can take microseconds while HBM is busy) overlap the wait instead
+    // of delaying the arrival.  The profiling hook p.stall_barrier (0: none)
+    // makes barrier number n unreachable, so that its bounded wait runs out
+    // and the launch ends with the timeout recorded.
+    __shared__ int s_ok;
+    auto barrier_arrive = [&]() {
         target += gridDim.x;
         ++n_barrier;
+        if (threadIdx.x == 0) grid_arrive(p.bar);
+    };
+    auto barrier_wait = [&]() {  // thread 0: result in s_ok
         const unsigned extra = n_barrier == p.stall_barrier ? 1u : 0u;
-        if (!grid_barrier(p.bar, target + extra, p.err, p.wait_ns)) return false;
+        s_ok = grid_wait(p.bar, target + extra, p.err, p.wait_ns) ? 1 : 0;
         // every CTA has read the sequence number before the first barrier
-        if (n_barrier == 1 && blockIdx.x == 0 && threadIdx.x == 0) *p.seq = s_seq + 1u;
-        return true;
+        if (s_ok && n_barrier == 1 && blockIdx.x == 0) *p.seq = s_seq + 1u;
     };
     Pipe pp{full, empty, acc_full, acc_empty, s_tmem, 0u, 0u, 0u, 0u, 0};
     bool prefetched = false;
@@ -1341,7 +1341,8 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         const FwdOp& op = s_op[o & 1];
         const int type = op.type;
         bool ok = true;
-        unsigned long long* ct = (p.trace && o == p.trace_op) ? p.trace + kTraceCtas + blockIdx.x * 8 : nullptr;
+        unsigned long long* ct = (p.trace && o == (p.trace_op & 0xffff)) ? p.trace + kTraceCtas + blockIdx.x * 8 : nullptr;
+        const bool ut_cta = ct && (int)blockIdx.x == (p.trace_op >> 16);  // the CTA whose units are stamped
         if (ct && threadIdx.x == 0) ct[0] = globaltimer();
         // the next op's arguments: the producer warp copies them (16 bytes a
         // lane, asynchronously) into their slot, which held op o-1, while op
@@ -1359,46 +1360,59 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         bool early = false;  // producer: the next projection's weights already requested
         if (is_gemm(type)) {
             ok = gemm_op<R>(op.g, epi_of(type), p.M, pos0, prefetched, smem, r_s, pp, (s_seq << 10) | (unsigned)o, p.err,
-                            (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr, ct);
+                            ut_cta ? p.trace + kTraceUnits : nullptr, ct);
         } else if (type == OP_EMBED) {
             embed_op(p, pos0);
         } else {
-            // attention: segment partials; then, while the grid gathers, the
-            // producer requests the next projection's first weights (the ring
-            // is free again), and after the barrier every CTA combines a share
-            // of the partials
+            // attention: segment partials; a grid barrier; then every CTA
+            // combines a share of the partials.  Between arriving and passing,
+            // the producer requests the next projection's first weights (the
+            // ring is free again); the consumers do not wait for that.
             ok = attn_op<R, HD>(op.at, p.M, pos0, smem, pp, p.err, ct, attn_pre,
-                                (ct && blockIdx.x == 0) ? p.trace + kTraceUnits : nullptr);
+                                ut_cta ? p.trace + kTraceUnits : nullptr);
+            if (__syncthreads_or(!ok)) {  // (uniform)
+                failed = true;
+                break;
+            }
+            if (ct && threadIdx.x == 0) ct[2] = globaltimer();
+            barrier_arrive();
             if (plane >= 0) {
                 asm volatile("cp.async.wait_all;" ::: "memory");
                 __syncwarp();
             }
-            if (plane == 0 && nx && ok && is_gemm(nx->type)) {
+            if (plane == 0 && nx && is_gemm(nx->type)) {
                 ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err);
                 early = true;
             }
-            if (!ok) s_fail = 1;
-            __syncthreads();
-            if (s_fail) {
-                failed = true;
-                break;
+            if (threadIdx.x < kConsumers) {  // (the producer and MMA warps go on to the op's end)
+                if (threadIdx.x == 0) {
+                    barrier_wait();
+                    if (ct) ct[7] = globaltimer();
+                }
+                consumer_sync();
+                if (s_ok) attn_combine<HD>(op.at, p.M, pos0);
+                else ok = false;
             }
-            if (!barrier_next()) {
-                failed = true;
-                break;
-            }
-            attn_combine<HD>(op.at, p.M, pos0);
         }
         if (ct && threadIdx.x == 0) ct[3] = globaltimer();
+        // the end of op o in this CTA (its stores ordered before thread 0's
+        // arrival); the last op needs no grid barrier
+        if (__syncthreads_or(!ok)) {
+            failed = true;
+            break;
+        }
+        if (ct && threadIdx.x == 0) ct[4] = globaltimer();
+        if (has_nx) barrier_arrive();
         // next op: visible to the producer warp now, to every thread after
-        // the CTA barrier below
+        // the CTA barrier below; the producer requests its first inputs that
+        // do not depend on op o while the grid gathers
         if (plane >= 0) {
             asm volatile("cp.async.wait_all;" ::: "memory");
             __syncwarp();
         }
         prefetched = false;
         attn_pre = 0;
-        if (plane == 0 && nx && ok) {
+        if (plane == 0 && nx) {
             if (is_gemm(nx->type)) {
                 if (!early) ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err);
                 prefetched = true;
@@ -1407,18 +1421,10 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
                 ok = attn_pre >= 0;
             }
         }
-        if (!ok) s_fail = 1;
-        __syncthreads();
-        if (s_fail) {
+        if (has_nx && threadIdx.x == 0) barrier_wait();
+        if (__syncthreads_or(!ok || (has_nx && threadIdx.x == 0 && !s_ok))) {
             failed = true;
             break;
-        }
-        if (ct && threadIdx.x == 0) ct[4] = globaltimer();
-        if (o + 1 < p.n_ops) {
-            if (!barrier_next()) {
-                failed = true;
-                break;
-            }
         }
         if (ct && threadIdx.x == 0) ct[5] = globaltimer();
         if (p.trace && blockIdx.x == 0 && threadIdx.x == 0) p.trace[o + 1] = globaltimer();

@@ -156,12 +156,11 @@ struct FwdParams {
     unsigned* seq;        // forward sequence number (tags split-K partials; +1 per launch)
     int* err;             // device error code
     // Profiling hook: nullptr, or globaltimer stamps: [0, n_ops] start, end of
-    // op o (CTA 0); [1024, 1280) CTA 0's first 64 units of op trace_op (producer
-    // issue, data ready, MMA done, flush done); [1280, 1280 + 8 * grid) per CTA,
-    // op trace_op: start, first data ready, last MMA done, work done, barrier
-    // arrive, barrier release, number of units, 0.
+    // op o (CTA 0); [1024, 1280) the first 64 units (or 31 attention items) of
+    // op trace_op & 0xffff on CTA trace_op >> 16; [1280, 1280 + 8 * grid) per
+    // CTA, op trace_op & 0xffff: the 8 stamps ssd_debug_trace_forward lists.
     unsigned long long* trace;
-    int trace_op;
+    int trace_op;  // -1: none
     // Bounded waits: a grid barrier gives up after wait_ns (error recorded).
     // Test hook: stall_barrier = n > 0 makes the n-th grid barrier of the
     // launch unreachable (0 in every production launch).
