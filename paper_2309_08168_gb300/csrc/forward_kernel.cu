@@ -53,6 +53,9 @@ namespace ssd {
 namespace {
 
 constexpr unsigned long long kBarrierTimeoutNs = 2000000000ull;
+// A wait reads the shared error flag only after this long (20 us): until
+// then each poll is a single load.
+constexpr unsigned long long kErrPollAfterNs = 20000ull;
 // 8 consumer warps (epilogues, attention, embedding) + 1 producer warp (TMA)
 // + 1 MMA warp (tcgen05.mma issue, TMEM allocation)
 constexpr int kConsumers = 256;
@@ -86,15 +89,20 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
 __device__ __forceinline__ void grid_arrive(unsigned* bar) {
     asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(bar) : "memory");
 }
+// Each poll is one L2 round trip: the error flag (another CTA gave up) is
+// read only once the wait has lasted kErrPollAfterNs, so that a second load
+// does not double the poll period of ordinary waits.
 __device__ bool grid_wait(unsigned* bar, unsigned target, int* err, unsigned long long limit_ns) {
     const unsigned long long t0 = globaltimer();
     while (ld_acquire(bar) < target) {
-        if (*(volatile int*)err) return false;
-        if (globaltimer() - t0 > limit_ns) {
-            atomicCAS(err, 0, kDevErrTimeout);
-            return false;
+        const unsigned long long dt = globaltimer() - t0;
+        if (dt > kErrPollAfterNs) {
+            if (*(volatile int*)err) return false;
+            if (dt > limit_ns) {
+                atomicCAS(err, 0, kDevErrTimeout);
+                return false;
+            }
         }
-        __nanosleep(32);
     }
     return true;
 }
@@ -169,13 +177,13 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, unsigned parity) {
     return ok != 0;
 }
 // bounded wait: false after kWaitTimeoutNs (timeout recorded), or once it has
-// waited 20 us while another thread has already recorded an error
+// waited kErrPollAfterNs while another thread has already recorded an error
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, unsigned parity, int* err) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = globaltimer();
     while (!mbar_try_wait(bar, parity)) {
         const unsigned long long dt = globaltimer() - t0;
-        if (dt > 20000ull && *(volatile int*)err) return false;
+        if (dt > kErrPollAfterNs && *(volatile int*)err) return false;
         if (dt > kWaitTimeoutNs) {
             atomicCAS(err, 0, kDevErrTimeout);
             return false;
@@ -443,8 +451,9 @@ __device__ __forceinline__ void advance_full(Pipe& pp, int n) {
 
 // Producer: requests the weights of this CTA's first S units of a projection
 // before the grid barrier (they do not depend on the previous op).
+// n_pre: how many (at most the ring's depth) are requested.
 template <int R>
-__device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, Pipe& pp, int* err) {
+__device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, Pipe& pp, int* err, int n_pre) {
     constexpr int S = GemmSmem<R>::S;
     int u_begin, n_my;
     my_units(a.n_units, &u_begin, &n_my);
@@ -452,7 +461,7 @@ __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, P
     if (threadIdx.x == kConsumers) {
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         prefetch_tmap(a.tm_x[plane_cls(R)]);
-        for (int s = 0; s < S && s < n_my && ok; ++s) {
+        for (int s = 0; s < S && s < n_pre && s < n_my && ok; ++s) {
             ok = mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err);
             if (!ok) break;
             pp.pphase ^= 1u << s;
@@ -472,7 +481,7 @@ __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, P
 // issue, MMAs issued, 0, segment flush done); ct: nullptr, or this CTA's op
 // stamps (FwdParams::trace) - profiling aids.
 template <int R>
-__device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefetched, unsigned char* smem,
+__device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, int n_pre, unsigned char* smem,
                         float* r_s, Pipe& pp, unsigned tag, int* err, unsigned long long* ut,
                         unsigned long long* ct) {
     using L = GemmSmem<R>;
@@ -487,13 +496,14 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 
     if (threadIdx.x >= kConsumers && threadIdx.x < kConsumers + 32) {  // producer warp
         if (threadIdx.x != kConsumers) return true;
+        if (ut) ut[2] = globaltimer();
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         asm volatile("fence.proxy.async.global;" ::: "memory");  // inputs written by the previous op
         for (int i = 0; i < n_my; ++i) {
             const int s = i % S;
             unsigned char* st = smem + s * L::STAGE;
             if (ut && i < 64) ut[i * 4 + 0] = globaltimer();
-            if (!(prefetched && i < S)) {
+            if (i >= n_pre) {  // (the first n_pre units' weights were requested before the op)
                 if (!mbar_wait(pp.empty + s, (pp.pphase >> s) & 1u, err)) return false;
                 pp.pphase ^= 1u << s;
                 tma_weights<R>(a, epi, u_begin + i, st, pp.full + s);
@@ -618,13 +628,14 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
                         if (ready) break;
                         const unsigned long long now = globaltimer();
                         if (t_wait == 0) t_wait = now;
-                        if (*(volatile int*)err) { ok = false; break; }
-                        if (now - t_wait > kBarrierTimeoutNs) {
-                            atomicCAS(err, 0, kDevErrTimeout);
-                            ok = false;
-                            break;
+                        if (now - t_wait > kErrPollAfterNs) {
+                            if (*(volatile int*)err) { ok = false; break; }
+                            if (now - t_wait > kBarrierTimeoutNs) {
+                                atomicCAS(err, 0, kDevErrTimeout);
+                                ok = false;
+                                break;
+                            }
                         }
-                        __nanosleep(64);
 #pragma unroll
                         for (int q = 0; q < QB; ++q)
 #pragma unroll
@@ -754,13 +765,14 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
                     if (ready) break;
                     const unsigned long long now = globaltimer();
                     if (t_wait == 0) t_wait = now;
-                    if (*(volatile int*)err) { ok = false; break; }
-                    if (now - t_wait > kBarrierTimeoutNs) {
-                        atomicCAS(err, 0, kDevErrTimeout);
-                        ok = false;
-                        break;
+                    if (now - t_wait > kErrPollAfterNs) {
+                        if (*(volatile int*)err) { ok = false; break; }
+                        if (now - t_wait > kBarrierTimeoutNs) {
+                            atomicCAS(err, 0, kDevErrTimeout);
+                            ok = false;
+                            break;
+                        }
                     }
-                    __nanosleep(64);
 #pragma unroll
                     for (int q = 0; q < QB; ++q)
 #pragma unroll
@@ -845,23 +857,23 @@ __device__ bool gemm_op(const GemmArgs& a, int epi, int M, int pos0, bool prefet
 }
 
 // ---------------------------------------------------------------------------
-// attention op: items (KV head, 256-position segment), through the TMA ring
+// attention op: items (KV head, vector group, 128-position segment), through
+// the TMA ring
 // ---------------------------------------------------------------------------
 // A segment is kAttnSegChunks absolute 64-position chunks; the producer thread
 // requests each chunk's K and V rows (TMA, 128-byte swizzle) into consecutive
-// ring stages, and after the CTA's last chunk it goes on to prefetch the next
-// projection's weights.  The consumers hold a segment's stages at once and,
-// for its G * M query vectors v (G query heads of the KV head, M rows), in
-// passes of up to VG vectors: scores (one thread per (v, position)), softmax
-// over the segment (one warp per v), P V (eight threads per (v, 8 dims),
-// interleaved positions, fixed shuffle tree); the partial (o, max, sum) of the segment goes to
-// global memory.  After its items, a CTA adds its count to each KV head's
-// counter; the last arrival combines the segment partials of that head in
-// segment order (flash-decoding style split of the softmax).  Every reduction
-// has a fixed order that depends only on the row's own position, not on M.
+// ring stages.  An item is one segment of one KV head for a group of up to 16
+// of its G * M query vectors (G query heads of the KV head, M rows): scores
+// and P V on tensor cores (fp16 hi + lo operands, fp32 accumulators), the
+// softmax over the segment from the score accumulators; the partial (o, max,
+// sum) of the segment goes to global memory.  Items run segment fastest, so a
+// CTA's consecutive items share their q.  After a grid barrier every CTA
+// combines a share of the (KV head, vector) partials in segment order
+// (flash-decoding style split of the softmax).  Every reduction has a fixed
+// order that depends only on the row's own position, not on M.
 struct AttnRange {
     int n_ch, n_seg, n_vg;  // chunks, segments per KV head, groups of 16 query vectors
-    int i_begin, i_end;     // this CTA's items (KV head, segment, vector group), group fastest
+    int i_begin, i_end;     // this CTA's items (KV head, vector group, segment), segment fastest
 };
 __device__ __forceinline__ AttnRange attn_range(const AttnArgs& a, int M, int pos0) {
     constexpr int S = kAttnSegChunks;
@@ -886,7 +898,7 @@ __device__ int attn_produce(const AttnArgs& a, const AttnRange& ar, int pos0, un
     constexpr int S = L::S, SC = kAttnSegChunks;
     int i = 0;
     for (int it = ar.i_begin; it < ar.i_end; ++it) {
-        const int hs = it / ar.n_vg, kvh = hs / ar.n_seg, c0 = (hs - kvh * ar.n_seg) * SC;
+        const int hv = it / ar.n_seg, kvh = hv / ar.n_vg, c0 = (it - hv * ar.n_seg) * SC;
         for (int c = c0; c < min(c0 + SC, ar.n_ch); ++c, ++i) {
             if (i < i_from) continue;
             if (i >= i_limit || (old_only && (c + 1) * kAttnChunk > pos0)) return i;
@@ -934,7 +946,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
         if (threadIdx.x == kConsumers + 32) {
             int n = 0;
             for (int it = ar.i_begin; it < ar.i_end; ++it) {
-                const int sg = (it / ar.n_vg) % ar.n_seg;
+                const int sg = it % ar.n_seg;
                 n += min(SC, ar.n_ch - sg * SC);
             }
             advance_full<S>(pp, n);
@@ -967,8 +979,8 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
     };
     for (int it = ar.i_begin; it < ar.i_end; ++it) {
         stamp(it, 0);
-        const int hs = it / ar.n_vg, vg = it - hs * ar.n_vg;
-        const int kvh = hs / ar.n_seg, sg = hs - kvh * ar.n_seg, t0 = sg * SP;
+        const int hv = it / ar.n_seg, sg = it - hv * ar.n_seg, t0 = sg * SP;
+        const int kvh = hv / ar.n_vg, vg = hv - kvh * ar.n_vg;
         const int n_u = min(SC, ar.n_ch - sg * SC);  // chunks of this segment
         const int v0 = vg * VG, nv = min(VG, NV - v0);
         float* part = a.part + ((size_t)kvh * a.n_chunks + sg) * NV * part_v;
@@ -1028,6 +1040,9 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
             const int p0 = warp * 16, j = p0 / kAttnChunk;
             float c[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
             if (j < n_u) {
+                // K q_hi and K q_lo in separate accumulators (two short
+                // dependency chains instead of one long one), added at the end
+                float cl[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
                 const unsigned char* kst = smem + ((i + j) % S) * L::STAGE;
                 const int t = (p0 % kAttnChunk) + (lane & 7) + 8 * ((lane >> 3) & 1);
                 const int qv = (lane & 7) + 8 * (lane >> 4), qk = ((lane >> 3) & 1) * 8;
@@ -1039,12 +1054,16 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
                     ldsm_x4(bh, qh + qv * QST + ks * 16 + qk);
                     ldsm_x4(bl, ql + qv * QST + ks * 16 + qk);
                     mma_f16_16816(c[0], af[0], af[1], af[2], af[3], bh[0], bh[1]);
-                    mma_f16_16816(c[0], af[0], af[1], af[2], af[3], bl[0], bl[1]);
+                    mma_f16_16816(cl[0], af[0], af[1], af[2], af[3], bl[0], bl[1]);
                     if (nv > 8) {  // vectors 8..15
                         mma_f16_16816(c[1], af[0], af[1], af[2], af[3], bh[2], bh[3]);
-                        mma_f16_16816(c[1], af[0], af[1], af[2], af[3], bl[2], bl[3]);
+                        mma_f16_16816(cl[1], af[0], af[1], af[2], af[3], bl[2], bl[3]);
                     }
                 }
+#pragma unroll
+                for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                    for (int x = 0; x < 4; ++x) c[nt][x] += cl[nt][x];
             }
             // C: rows = positions p0 + g (+8), columns = vectors 8 nt + 2 tg (+1)
 #pragma unroll
@@ -1113,7 +1132,9 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
         // transposed 8x8 loads), all 16 vectors (A = P hi, then lo); rows of
         // vectors past nv hold stale weights and are not stored
         if (warp * 16 < HD) {
+            // P_hi V and P_lo V in separate accumulators, added at the end
             float c[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+            float cl[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
             const int d = warp * 16 + 8 * (lane >> 4), bx = d >> 6, cc = (d & 63) >> 3;
             const int pv = (lane & 7) + 8 * ((lane >> 3) & 1), pk = (lane >> 4) * 8;
             for (int ks = 0; ks < n_u * (kAttnChunk / 16); ++ks) {
@@ -1124,9 +1145,13 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
                 ldsm_x4_t(bv, smem + ((i + j) % S) * L::STAGE + 16384 + bx * 8192 + tt * 128 + ((cc ^ (tt & 7)) << 4));
                 mma_f16_16816(c[0], ah[0], ah[1], ah[2], ah[3], bv[0], bv[1]);
                 mma_f16_16816(c[1], ah[0], ah[1], ah[2], ah[3], bv[2], bv[3]);
-                mma_f16_16816(c[0], al[0], al[1], al[2], al[3], bv[0], bv[1]);
-                mma_f16_16816(c[1], al[0], al[1], al[2], al[3], bv[2], bv[3]);
+                mma_f16_16816(cl[0], al[0], al[1], al[2], al[3], bv[0], bv[1]);
+                mma_f16_16816(cl[1], al[0], al[1], al[2], al[3], bv[2], bv[3]);
             }
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int x = 0; x < 4; ++x) c[nt][x] += cl[nt][x];
             // C: rows = vectors g (+8), columns = dims 16w + 8 nt + 2 tg (+1)
 #pragma unroll
             for (int nt = 0; nt < 2; ++nt)
@@ -1255,6 +1280,10 @@ __device__ void drain_before_exit() {
     __syncthreads();
 }
 
+// Units of the next projection whose weights the producer requests between
+// its CTA's arrival at an op boundary's grid barrier and the barrier's end.
+constexpr int kBoundaryPrefetch = 5;
+
 template <int R, int HD>
 __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams p) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -1333,7 +1362,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         if (s_ok && n_barrier == 1 && blockIdx.x == 0) *p.seq = s_seq + 1u;
     };
     Pipe pp{full, empty, acc_full, acc_empty, s_tmem, 0u, 0u, 0u, 0u, 0};
-    bool prefetched = false;
+    int n_pre = 0;  // producer: units of the op whose weights were requested before it
     bool failed = false;
     int attn_pre = 0;  // producer: K / V chunks of the next attention op requested early
     copy_op(p.ops, s_op);
@@ -1359,7 +1388,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
         const FwdOp* nx = has_nx ? s_op + ((o + 1) & 1) : nullptr;
         bool early = false;  // producer: the next projection's weights already requested
         if (is_gemm(type)) {
-            ok = gemm_op<R>(op.g, epi_of(type), p.M, pos0, prefetched, smem, r_s, pp, (s_seq << 10) | (unsigned)o, p.err,
+            ok = gemm_op<R>(op.g, epi_of(type), p.M, pos0, n_pre, smem, r_s, pp, (s_seq << 10) | (unsigned)o, p.err,
                             ut_cta ? p.trace + kTraceUnits : nullptr, ct);
         } else if (type == OP_EMBED) {
             embed_op(p, pos0);
@@ -1381,7 +1410,7 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
                 __syncwarp();
             }
             if (plane == 0 && nx && is_gemm(nx->type)) {
-                ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err);
+                ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err, GemmSmem<R>::S);
                 early = true;
             }
             if (threadIdx.x < kConsumers) {  // (the producer and MMA warps go on to the op's end)
@@ -1410,18 +1439,21 @@ __global__ void __launch_bounds__(kFwdThreads, 1) forward_kernel(const FwdParams
             asm volatile("cp.async.wait_all;" ::: "memory");
             __syncwarp();
         }
-        prefetched = false;
+        n_pre = 0;
         attn_pre = 0;
         if (plane == 0 && nx) {
             if (is_gemm(nx->type)) {
-                if (!early) ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err);
-                prefetched = true;
+                n_pre = (early || kBoundaryPrefetch > GemmSmem<R>::S) ? GemmSmem<R>::S : kBoundaryPrefetch;
+                if (!early) ok = gemm_prefetch<R>(nx->g, epi_of(nx->type), smem, pp, p.err, n_pre);
             } else if (nx->type == OP_ATTN) {
                 attn_pre = attn_prefetch<R, HD>(nx->at, p.M, pos0, smem, pp, p.err);
                 ok = attn_pre >= 0;
             }
         }
-        if (has_nx && threadIdx.x == 0) barrier_wait();
+        if (has_nx && threadIdx.x == 0) {
+            barrier_wait();
+            if (ct && is_gemm(type)) ct[7] = globaltimer();
+        }
         if (__syncthreads_or(!ok || (has_nx && threadIdx.x == 0 && !s_ok))) {
             failed = true;
             break;
