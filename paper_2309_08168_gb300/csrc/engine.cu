@@ -327,18 +327,14 @@ void set_x_maps(const ssd_handle* h, GemmArgs& a, int buf) {
 }
 
 // One projection op: fills the fields every projection shares.
-GemmArgs proj_args(ssd_handle* h, int N, int K, int n_tiles, const bf16* x_hi, const bf16* x_lo) {
+GemmArgs proj_args(ssd_handle* h, int N, int K, int n_tiles) {
     GemmArgs a{};
     a.N = N;
     a.K = K;
     a.n_tiles = n_tiles;
     a.n_chunks = (K + kFKC - 1) / kFKC;
-    a.wide = 1;
     a.n_units = n_tiles * a.n_chunks;
-    a.x_hi = x_hi;
-    a.x_lo = x_lo;
     a.partial = h->partial;
-    a.st = h->st;
     a.err = &h->st->err;
     a.inv_dim = 1.0f / (float)h->cfg.d_model;
     a.eps = h->cfg.rms_eps;
@@ -365,7 +361,7 @@ std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
             FwdOp q{};
             q.type = OP_QKV;
             GemmArgs& a = q.g;
-            a = proj_args(h, qd + 2 * kvd, d, (qd + 2 * kvd) / kFTile, h->xn_hi, h->xn_lo);
+            a = proj_args(h, qd + 2 * kvd, d, (qd + 2 * kvd) / kFTile);
             a.w0 = h->wq[l]; a.w1 = h->wk[l]; a.w2 = h->wv[l];
             a.tm_w[0] = h->tmaps + tmap_weight(l, 0);
             a.tm_w[1] = h->tmaps + tmap_weight(l, 1);
@@ -391,7 +387,7 @@ std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
             ops.push_back(at);
             FwdOp o{};
             o.type = OP_RESID;
-            o.g = proj_args(h, d, qd, d_tiles, h->at_hi, h->at_lo);
+            o.g = proj_args(h, d, qd, d_tiles);
             o.g.w0 = h->wo[l];
             o.g.tm_w[0] = h->tmaps + tmap_weight(l, 3);
             set_x_maps(h, o.g, 1);
@@ -402,7 +398,7 @@ std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
         if (run_m) {
             FwdOp gu{};
             gu.type = OP_SWIGLU;
-            gu.g = proj_args(h, 2 * c.ffn, d, (c.ffn + 63) / 64, h->xn_hi, h->xn_lo);
+            gu.g = proj_args(h, 2 * c.ffn, d, (c.ffn + 63) / 64);
             gu.g.w0 = h->w_gate[l]; gu.g.w1 = h->w_up[l];
             gu.g.tm_w[0] = h->tmaps + tmap_weight(l, 4);
             gu.g.tm_w[1] = h->tmaps + tmap_weight(l, 5);
@@ -412,7 +408,7 @@ std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
             ops.push_back(gu);
             FwdOp w{};
             w.type = OP_RESID;
-            w.g = proj_args(h, d, c.ffn, d_tiles, h->ac_hi, h->ac_lo);
+            w.g = proj_args(h, d, c.ffn, d_tiles);
             w.g.w0 = h->w_down[l];
             w.g.tm_w[0] = h->tmaps + tmap_weight(l, 6);
             set_x_maps(h, w.g, 2);
@@ -423,7 +419,7 @@ std::vector<FwdOp> build_ops(ssd_handle* h, bool draft) {
     }
     FwdOp lg{};
     lg.type = OP_LOGITS;
-    lg.g = proj_args(h, c.vocab, d, (c.vocab + kFTile - 1) / kFTile, h->xn_hi, h->xn_lo);
+    lg.g = proj_args(h, c.vocab, d, (c.vocab + kFTile - 1) / kFTile);
     lg.g.w0 = h->lm_head;
     lg.g.tm_w[0] = h->tmaps + 7 * c.n_layers;
     set_x_maps(h, lg.g, 0);

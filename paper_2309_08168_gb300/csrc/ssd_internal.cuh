@@ -62,18 +62,17 @@ struct GemmArgs {
     const bf16* w2;      // segment 2 (wv)
     int N;               // logical output rows
     int K;               // reduction length (row length of every segment)
-    int kc;              // k-chunk per CTA (multiple of 64)
-    int ksplit;          // ceil(K / kc)
+    int kc;              // gemm.cu: k-chunk per CTA (multiple of 64)
+    int ksplit;          // gemm.cu: ceil(K / kc)
     int n_tiles;         // row tiles
-    const float* x;      // activations [M][K] fp32 (split into bf16 hi + lo in the kernel)
-    int M;               // activation rows (1..16)
+    const float* x;      // gemm.cu: activations [M][K] fp32 (split into bf16 hi + lo in the kernel)
+    int M;               // gemm.cu: activation rows (1..16)
     float* partial;      // split-K partials: gemm.cu [ksplit][M][n_tiles*64] floats; forward
                          // kernel [n_tiles][n_chunks][16][128] tagged 64-bit words
-    unsigned* counters;  // gemm.cu: [n_tiles] arrival counters (left at zero); unused by the forward kernel
+    unsigned* counters;  // gemm.cu: [n_tiles] arrival counters (left at zero)
     // epilogue operands
     float* out_f32;      // EPI_LOGITS: [M][ldo]; EPI_RESID: residual h [M][ldo]
     int ldo;
-    float* out_act;      // EPI_SWIGLU: act [M][ffn]
     int ffn;
     // EPI_QKV
     int n_heads, n_kv_heads, head_dim, max_seq;
@@ -81,11 +80,7 @@ struct GemmArgs {
     f16* k_cache;        // this layer: [Hkv][max_seq][hd] fp16
     f16* v_cache;
     const float2* rope;  // [max_seq][hd/2] (cos, sin)
-    const DecodeState* st;  // pos0
-    int* err;            // device error flag (checked builds)
-    // streaming GEMM (gemm_stream.cu)
-    const bf16* x_hi;    // input planes [M][K]: bf16 hi = rn(v), lo = rn(v - hi)
-    const bf16* x_lo;
+    int* err;            // device error flag
     const float* ss_in;  // [M][ss_in_tiles] sums of squares of the pre-norm row (nullptr: no norm)
     int ss_in_tiles;
     float inv_dim, eps;  // RMSNorm scale of row m: rsqrt(sum(ss_in[m]) * inv_dim + eps)
@@ -99,7 +94,6 @@ struct GemmArgs {
     // {K, rows} with box {64, 128} (SwiGLU gate / up: {64, 64}), one copy per
     // 64-wide k box of a unit; x maps view the planes as {K, 16, 2} with box
     // {64, R, 2}, one copy per k box.
-    int wide;            // (unused by the forward kernel)
     const void* tm_w[3];  // w0, w1, w2
     const void* tm_x[kPlaneClasses];  // input planes for R = 1 | 4 | 8 | 12 | 16
 };
