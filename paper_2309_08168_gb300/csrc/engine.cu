@@ -115,7 +115,7 @@ struct ssd_handle {
     float* p_rows = nullptr;
     float* q_rows = nullptr;
     float* partial = nullptr;
-    unsigned* counters = nullptr;  // [attention kv heads | accept] arrival counters
+    unsigned* counters = nullptr;  // [4]: the acceptance kernels' arrival counter (+ spare words)
     float* attn_part = nullptr;
     int n_chunks = 0;
     float2* rope = nullptr;
@@ -487,7 +487,7 @@ double forward_weight_bytes(const ssd_handle* h, bool draft, bool gemm_only) {
     return b;
 }
 
-unsigned* accept_counter(ssd_handle* h) { return h->counters + h->cfg.n_kv_heads; }
+unsigned* accept_counter(ssd_handle* h) { return h->counters; }
 
 int step_launches(ssd_handle* h, int kind, int M, int mode, int* n_launch) {
     const int V = h->cfg.vocab;
@@ -700,8 +700,8 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
         (rc = dalloc(h, &h->p_rows, (size_t)kMaxRows * V, &B)) ||
         (rc = dalloc(h, &h->q_rows, (size_t)kMaxRows * V, &B)) ||
         (rc = dalloc(h, &h->partial, 2 * part, &B)) ||  // tagged 64-bit words in the forward kernel
-        (rc = dalloc(h, &h->counters, (size_t)c.n_kv_heads + 4, &B)) ||
-        (rc = dalloc(h, &h->attn_part, (size_t)c.n_kv_heads * h->n_chunks * G * kMaxRows * (HD + 2), &B)) ||
+        (rc = dalloc(h, &h->counters, (size_t)4, &B)) ||
+        (rc = dalloc(h, &h->attn_part, (size_t)c.n_kv_heads * h->n_chunks * G * kMaxRows * attn_part_floats((int)HD), &B)) ||
         (rc = dalloc(h, &h->rope, (size_t)c.max_seq * (HD / 2), &B)) ||
         (rc = dalloc(h, &h->tok, (size_t)c.max_seq + kMaxRows, &B)) ||
         (rc = dalloc(h, &h->out, (size_t)c.max_seq, &B)) || (rc = dalloc(h, &h->argbuf, 32, &B)) ||
@@ -735,7 +735,7 @@ int ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, s
         cudaError_t e = cudaMemcpy(h->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice);
         if (e != cudaSuccess) return bail(fail(SSD_ERR_CUDA, std::string("rope table: ") + cudaGetErrorString(e)));
     }
-    cudaError_t e = cudaMemsetAsync(h->counters, 0, ((size_t)c.n_kv_heads + 4) * sizeof(unsigned), h->stream);
+    cudaError_t e = cudaMemsetAsync(h->counters, 0, 4 * sizeof(unsigned), h->stream);
     if (e == cudaSuccess) e = cudaMemsetAsync(h->st, 0, sizeof(DecodeState), h->stream);
     // barrier counter and forward sequence number; split-K slots hold no
     // valid tag (a tag is never 0: GEMM ops have an op index >= 1)
@@ -830,7 +830,7 @@ int ssd_prefill(ssd_handle* h, const int32_t* prompt, int n_prompt) {
     // the acceptance kernels' arrival counter is left at zero by every
     // completed launch; after a failed one it may not be, so a new prompt
     // starts from clean counters
-    CUDA_TRY(cudaMemsetAsync(h->counters, 0, ((size_t)h->cfg.n_kv_heads + 4) * sizeof(unsigned), h->stream),
+    CUDA_TRY(cudaMemsetAsync(h->counters, 0, 4 * sizeof(unsigned), h->stream),
              "counter reset");
     if (n_prompt > 1)
         CUDA_TRY(cudaMemcpyAsync(h->tok, prompt, sizeof(int) * (n_prompt - 1), cudaMemcpyHostToDevice, h->stream),

@@ -968,7 +968,7 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
     __half* pl = ph + VG * PST;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, tg = lane & 3;
-    const size_t part_v = HD + 2;  // floats per partial: o[HD], max, sum
+    constexpr size_t part_v = attn_part_floats(HD);  // floats per partial: o[HD], max, sum, pad
     bool ok = true;
     int i = 0;       // ring position within the op
     int q_key = -1;  // (KV head, vector group) whose q is in shared memory
@@ -1176,54 +1176,77 @@ __device__ bool attn_op(const AttnArgs& a, int M, int pos0, unsigned char* smem,
 // Second phase of attention, after a grid barrier (the segment partials of
 // every CTA are visible): the partials of each (KV head, query vector) are
 // combined in segment order - row m uses segments 0 .. (pos0 + m) / SP - and
-// written as the bf16 hi / lo planes of the attention output.  One warp (half
-// a warp at head_dim 64) per vector, 4 dims per thread (coalesced loads), the
-// vectors spread round-robin over the warps of all CTAs, so the combine
-// costs about two dependent L2 round trips whatever the number of vectors
-// and segments, and no SM carries much of its traffic.
+// written as the bf16 hi / lo planes of the attention output.  One warp per
+// 64 dims of a vector (2 dims per lane), spread round-robin over the warps of
+// all CTAs.  Per batch of up to kCombineBatch segments a lane loads its dims of
+// every segment and lane j the (max, sum) of segment j, all at once (one L2
+// round trip per batch: one for contexts up to 2048 positions); the batch
+// maximum and the sum of the weighted sums are shuffle trees, the weighted
+// dims are added in segment order, and batches fold into running sums scaled
+// to the running maximum.  The order depends only on the row's position.
+constexpr int kCombineBatch = 16;
 template <int HD>
 __device__ void attn_combine(const AttnArgs& a, int M, int pos0) {
     if (threadIdx.x >= kConsumers) return;
-    constexpr int SP = kAttnSegChunks * kAttnChunk, HD4 = HD / 4, VPW = 32 / HD4;  // vectors per warp
+    constexpr int SP = kAttnSegChunks * kAttnChunk, HALVES = HD / 64, B = kCombineBatch;
+    static_assert(B <= 32, "one lane per segment of a batch");
     const int G = a.n_heads / a.n_kv_heads, NV = G * M;
-    const size_t part_v = HD + 2;                  // floats per partial: o[HD], max, sum
-    const size_t qs_stride = (size_t)NV * part_v;  // next segment of the same vector
-    const int n_vec = a.n_kv_heads * NV;
+    constexpr size_t part_v = attn_part_floats(HD);  // floats per partial: o[HD], max, sum, pad
+    const size_t qs_stride = (size_t)NV * part_v;    // next segment of the same vector
+    const int n_work = a.n_kv_heads * NV * HALVES;   // (vector, 64 dims) per warp
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int n_warps = gridDim.x * (kConsumers / 32);
-    // warp-major over the CTAs: the first vectors go to warp 0 of every CTA
-    for (int gv = (warp * gridDim.x + blockIdx.x) * VPW + lane / HD4; gv < n_vec; gv += n_warps * VPW) {
+    // warp-major over the CTAs: the first work items go to warp 0 of every CTA
+    for (int wk = warp * gridDim.x + blockIdx.x; wk < n_work; wk += n_warps) {
+        const int gv = wk / HALVES, hf = wk - gv * HALVES;
         const int kvh = gv / NV, v = gv - kvh * NV;
-        const int e = (lane % HD4) * 4;
+        const int e = hf * 64 + 2 * lane;
         const int m = v / G, gi = v - m * G;
         const int nsg = (pos0 + m) / SP + 1;
         const float* pv = a.part + (size_t)kvh * a.n_chunks * qs_stride + (size_t)v * part_v;
-        float mx = -INFINITY;
-#pragma unroll 8
-        for (int q = 0; q < nsg; ++q) mx = fmaxf(mx, __ldcg(pv + q * qs_stride + HD));
-        float l = 0.f, o0 = 0.f, o1 = 0.f, o2 = 0.f, o3 = 0.f;
-#pragma unroll 8
-        for (int q = 0; q < nsg; ++q) {
-            const float* pq = pv + q * qs_stride;
-            const float mq = __ldcg(pq + HD);
-            const float f = mq == -INFINITY ? 0.f : expf(mq - mx);  // empty segments hold o = 0
-            const float2 oa = __ldcg(reinterpret_cast<const float2*>(pq + e));
-            const float2 ob = __ldcg(reinterpret_cast<const float2*>(pq + e + 2));
-            l += f * __ldcg(pq + HD + 1);
-            o0 += f * oa.x;
-            o1 += f * oa.y;
-            o2 += f * ob.x;
-            o3 += f * ob.y;
+        float mx = -INFINITY, l = 0.f, o0 = 0.f, o1 = 0.f;
+        for (int q0 = 0; q0 < nsg; q0 += B) {
+            const int nb = min(B, nsg - q0);
+            float2 ml = make_float2(-INFINITY, 0.f);  // (max, sum) of segment q0 + lane
+            if (lane < nb) ml = __ldcg(reinterpret_cast<const float2*>(pv + (size_t)(q0 + lane) * qs_stride + HD));
+            float2 ov[B];
+#pragma unroll
+            for (int j = 0; j < B; ++j) {
+                ov[j] = make_float2(0.f, 0.f);
+                if (j < nb) ov[j] = __ldcg(reinterpret_cast<const float2*>(pv + (size_t)(q0 + j) * qs_stride + e));
+            }
+            float bm = ml.x;
+#pragma unroll
+            for (int off = 16; off; off >>= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, off));
+            bm = fmaxf(bm, mx);
+            // empty segments (and lanes past the batch) hold max -inf, o = 0
+            const float r = mx == -INFINITY ? 0.f : expf(mx - bm);
+            const float f = ml.x == -INFINITY ? 0.f : expf(ml.x - bm);
+            float fl = f * ml.y;
+#pragma unroll
+            for (int off = 16; off; off >>= 1) fl += __shfl_xor_sync(0xffffffffu, fl, off);
+            l = l * r + fl;
+            o0 *= r;
+            o1 *= r;
+#pragma unroll
+            for (int j = 0; j < B; ++j) {
+                const float fj = __shfl_sync(0xffffffffu, f, j);
+                o0 += fj * ov[j].x;
+                o1 += fj * ov[j].y;
+            }
+            mx = bm;
         }
         const float inv = 1.f / l;
         const size_t at = (size_t)m * a.n_heads * HD + (size_t)(kvh * G + gi) * HD + e;
-        const float val[4] = {o0 * inv, o1 * inv, o2 * inv, o3 * inv};
-#pragma unroll
-        for (int x = 0; x < 4; ++x) {
-            const bf16 vh = __float2bfloat16_rn(val[x]);
-            a.out_hi[at + x] = vh;
-            a.out_lo[at + x] = __float2bfloat16_rn(val[x] - __bfloat162float(vh));
-        }
+        const float v0 = o0 * inv, v1 = o1 * inv;
+        const bf16 h0 = __float2bfloat16_rn(v0), h1 = __float2bfloat16_rn(v1);
+        __nv_bfloat162 hi, lo;
+        hi.x = h0;
+        hi.y = h1;
+        lo.x = __float2bfloat16_rn(v0 - __bfloat162float(h0));
+        lo.y = __float2bfloat16_rn(v1 - __bfloat162float(h1));
+        *reinterpret_cast<__nv_bfloat162*>(a.out_hi + at) = hi;
+        *reinterpret_cast<__nv_bfloat162*>(a.out_lo + at) = lo;
     }
 }
 

@@ -102,6 +102,10 @@ struct GemmArgs {
 // attention (decode / verification over the KV cache, split into absolute
 // 64-position chunks, fixed-order combine)
 // ---------------------------------------------------------------------------
+// floats per attention segment partial: o[hd], max, sum, and 2 of padding so
+// that every partial starts on a 16-byte boundary (vector loads in the combine)
+__host__ __device__ constexpr int attn_part_floats(int hd) { return hd + 4; }
+
 struct AttnArgs {
     const float* q;      // [M][H*hd]
     // TMA maps of the whole K / V cache viewed as {hd, max_seq, L * Hkv} fp16,
@@ -111,7 +115,7 @@ struct AttnArgs {
     int kv_z0;
     bf16* out_hi;        // [M][H*hd] output planes: hi = rn(o), lo = rn(o - hi)
     bf16* out_lo;
-    float* part;         // segment partials [Hkv][n_chunks][G*M][hd + 2]: o[hd], max, sum
+    float* part;         // segment partials [Hkv][n_chunks][G*M][attn_part_floats(hd)]: o[hd], max, sum, 2 pad
     int M, n_heads, n_kv_heads, head_dim, max_seq, n_chunks;
     float scale;         // 1/sqrt(hd)
     const DecodeState* st;
