@@ -63,7 +63,7 @@ struct TcArgs {
     int rows;              // valid token rows
     int K;
     int n_kb;              // ceil(K / 64)
-    int n_tiles;           // column tiles (gridDim.x)
+    int n_tiles;           // column tiles (gridDim.y)
     int N;                 // valid output columns (STORE / RESID: width of out)
     float* out;            // STORE: [rows][ldo] fp32; RESID: residual h [rows][ldo] (+= D)
     int ldo;
@@ -218,7 +218,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const TcArgs a) {
     __shared__ int s_fail;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int tile = blockIdx.x, m0 = blockIdx.y * kBM;
+    // row tiles fastest: the CTAs that share a weight tile run together, so
+    // each weight tile is read from DRAM once and from L2 by the other rows
+    const int tile = blockIdx.y, m0 = blockIdx.x * kBM;
     if (threadIdx.x == 0) {
         s_fail = 0;
         for (int s = 0; s < kStages; ++s) {
@@ -380,7 +382,7 @@ inline int tc_configure() {
 
 template <int EPI>
 inline int tc_launch(const TcArgs& a, int row_tiles, cudaStream_t s) {
-    tc_gemm_kernel<EPI><<<dim3(a.n_tiles, row_tiles), kThreads, kSmemBytes, s>>>(a);
+    tc_gemm_kernel<EPI><<<dim3(row_tiles, a.n_tiles), kThreads, kSmemBytes, s>>>(a);
     return (int)cudaGetLastError();
 }
 
