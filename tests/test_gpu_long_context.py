@@ -9,7 +9,8 @@ the GPU logits are compared with the fp64 oracle, element by element at
 
   * tiny (4 layers, d 256): 300-token prompt, verification over 1, 5, 9, 13
     and 16 rows (every input-plane class) and the draft rows one by one;
-    rows straddling the segment boundaries at 128 and 256;
+    rows straddling the segment boundaries at 128 and 256; a 2070-token
+    prompt, past the 16 segments the combine folds in one batch;
   * LLaMA-2-7B widths (2 layers, 32 heads): 400-token prompt, 9 rows;
   * LLaMA-2-70B widths (2 layers, GQA 64 query / 8 KV heads): 300-token
     prompt, 9 rows, so 72 query vectors of each KV head meet several
@@ -73,6 +74,17 @@ def test_tiny_three_segments(tiny_setup, n_rows):
     got_d, ref_d, got_v, ref_v = draft_then_verify(w, hw, dw, 300, n_rows, seed=21, max_seq=320)
     assert_logits_close(got_v, ref_v, f"tiny verify M={n_rows} at 299")
     assert_logits_close(got_d, ref_d, f"tiny draft rows at 299")
+
+
+def test_tiny_beyond_one_combine_batch(tiny_setup):
+    """Contexts past 16 segments (2048 positions): the combine folds a second
+    batch of segment partials into running sums rescaled to the new maximum.
+    A 2070-token prompt (two prefill chunks), 9 verification rows and the
+    draft rows at positions 2069 .. 2077 (17 segments)."""
+    w, hw, dw = tiny_setup
+    got_d, ref_d, got_v, ref_v = draft_then_verify(w, hw, dw, 2070, 9, seed=51, max_seq=2100)
+    assert_logits_close(got_v, ref_v, "tiny verify M=9 at 2069")
+    assert_logits_close(got_d, ref_d, "tiny draft rows at 2069")
 
 
 @pytest.mark.parametrize("P", [125, 253])
