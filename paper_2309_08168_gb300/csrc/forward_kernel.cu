@@ -7,9 +7,9 @@
 // the step.  Instead one CTA per SM walks the forward's op list
 //     embed -> [QKV -> attention -> O] -> [gate/up -> down] -> ... -> lm_head
 // (sublayers in the skip set z are simply absent from the draft's list,
-// Sec. 3.2 / 3.3) with a grid barrier between dependent ops.  Before entering
-// a barrier every CTA already requests the weights of its first units of the
-// next projection (they do not depend on the previous op), so the barrier's
+// Sec. 3.2 / 3.3) with a grid barrier between dependent ops.  Once a CTA has
+// arrived at a barrier it requests the weights of its first units of the next
+// projection (they do not depend on the previous op), so the barrier's
 // latency overlaps HBM streaming.  Every wait is bounded: a barrier that does
 // not complete within ~2 s records an error code and the CTAs return.
 //
@@ -17,7 +17,7 @@
 // residual add, gate/up with SwiGLU, lm_head) run on the 5th-generation
 // tensor cores: work unit = 128-row tile x 128-wide k chunk (32 KB of
 // weights), each CTA owns an equal contiguous range of units in tile-major
-// order, streamed by TMA (128-byte swizzle) through a 4-5 stage ring; one
+// order, streamed by TMA (128-byte swizzle) through a 5-stage ring; one
 // thread of the MMA warp issues tcgen05.mma kind::f16 per unit (M = 128 weight
 // rows, N = the activation rows as bf16 hi + lo planes, ~16 mantissa bits of
 // the fp32 activations) into a TMEM accumulator and releases the stage with
@@ -31,9 +31,9 @@
 // of h * g_next and per-128-column sums of h^2, the consumer scales row m by
 // rsqrt(mean(h^2) + eps) in its epilogue (W (h g r) = r W (h g)).
 //
-// Attention: items = (KV head, absolute 128-position segment, group of 16
-// query vectors); the partial softmax of a row over a segment depends only on
-// the row and the segment.  After a grid barrier every CTA combines a share
+// Attention: items = (KV head, group of 16 query vectors, absolute
+// 128-position segment); the partial softmax of a row over a segment depends
+// only on the row and the segment.  After a grid barrier every CTA combines a share
 // of the (KV head, query vector) outputs over their segments in segment
 // order.
 //
@@ -432,7 +432,7 @@ struct Pipe {
     uint64_t* full;     // [stages] TMA completion (count 1: the producer's arrive)
     uint64_t* empty;    // [stages] stage released (count 1: tcgen05.commit, or consumer thread 0)
     uint64_t* acc_full;   // [2] accumulator complete (tcgen05.commit)
-    uint64_t* acc_empty;  // [2] accumulator read by the consumers (thread 0)
+    uint64_t* acc_empty;  // [2] accumulator read by the consumers (count 8: one arrival per consumer warp)
     uint32_t tmem;      // TMEM base address (two accumulators of kTmemCols / 2 columns)
     unsigned pphase;
     unsigned cphase;
@@ -476,7 +476,8 @@ __device__ bool gemm_prefetch(const GemmArgs& a, int epi, unsigned char* smem, P
 //   MMA issuer (one thread of warp 9) runs tcgen05.mma per unit into the
 //     accumulator of the unit's tile segment;
 //   consumers (warps 0-7), per finished segment: TMEM -> hi + lo summed ->
-//     split-K exchange -> epilogue.
+//     split-K exchange -> epilogue (contributors and residual finalisers
+//     per warp from registers, the other finalisers through shared memory).
 // ut: nullptr, or [64][4] timestamps of this CTA's first units (producer
 // issue, MMAs issued, 0, segment flush done); ct: nullptr, or this CTA's op
 // stamps (FwdParams::trace) - profiling aids.
